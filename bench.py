@@ -1,0 +1,439 @@
+#!/usr/bin/env python3
+"""Benchmark of the PSS hashed shared-array embedding step on GB300.
+
+One step = the whole hot path over one batch: fused hash + gather + sum-pool
+forward, then the backward scatter fused with the optimizer update of the
+shared array.  Default workload: the Criteo-TB-shaped 10000x-compressed case
+(26 tables, ~195M ids capped at 40M per table, d = 128, M = 2.5M fp32,
+Z = 32, batch 65536, Zipf(1.05) ids, Adagrad).
+
+Prints ONE JSON line (rank 0).  ``--impl reference`` times the CPU oracle
+instead (the reference arm: a deliberately plain program).
+
+Usage:  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload tb]
+        torchrun --nproc-per-node N bench.py --gpus N ...   (independent replicas)
+"""
+from __future__ import annotations
+
+import argparse
+import datetime as _dt
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2207_10731_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "pooled lookups/sec and fused fwd+bwd+update GB/s vs HBM/L2 roofline, 1 GB300"
+UNIT = "lookups/s"
+WORKLOAD_DESC = {
+    "tb": "criteo-tb-shaped 10000x: 26 tables (log-uniform cards in [3,40M], ~195M ids), d=128, "
+          "M=2.5M fp32 (10 MB), Z=32, G=4, batch 65536, one Zipf(1.05) id per bag, Adagrad",
+    "kaggle": "criteo-kaggle-shaped: 26 tables (log-uniform cards in [3,10M]), d=16, M=1Mi fp32, "
+              "Z=32, G=4, batch 2048, one Zipf(1.05) id per bag, Adagrad",
+    "multihot": "multi-hot contention: 26 tables as criteo-tb, d=64, M=2.5M fp32, Z=32, G=4, "
+                "batch 16384, Poisson(20) bags, Zipf(1.2) ids, SGD",
+    "sweep": "criteo-tb shape with shared array M chosen by --M, Z=32, G=4, batch 65536, Adagrad",
+    "microbench": "paper micro-benchmark shape: 26 tables, d=128, M=2.5M, Z=32, batch 10240, "
+                  "all-ones upstream gradient, SGD",
+    "tiny": "tiny: 8 tables x 1000 ids, d=16, M=16384, Z=16, batch 256, SGD",
+}
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _kernel_sha():
+    h = hashlib.sha256()
+    for f in ("pss_kernels.cu", "pss_device.cuh"):
+        with open(os.path.join(ROOT, "paper_2207_10731_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def _traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if the kernel
+    source has not changed since it was captured."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            t = json.load(f)
+        e = t.get(f"{kernel}@{workload}")
+        if e and e.get("kernel_sha") == _kernel_sha():
+            return float(e["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples with their own timestamps."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.rows = []
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", gpu_id], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.th = threading.Thread(target=self._read, daemon=True)
+        self.th.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                ts = _dt.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                self.rows.append((ts, float(parts[1]), float(parts[2]), parts[4:8]))
+            except ValueError:
+                continue
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float):
+        if not self.rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "note": "nvidia-smi unavailable"}
+        inside = [r for r in self.rows if t0 <= r[0] <= t1]
+        note = "samples inside the timed region"
+        if not inside:
+            mid = 0.5 * (t0 + t1)
+            inside = sorted(self.rows, key=lambda r: abs(r[0] - mid))[:3]
+            note = "timed region shorter than the sampling period: nearest samples"
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i, v in enumerate(r[3]) if v == "Active"})
+        return {"sm_mhz": float(np.median([r[1] for r in inside])),
+                "sm_max_mhz": float(max(r[2] for r in inside)), "reasons": reasons,
+                "samples": len(inside), "note": note}
+
+
+def _gpu_id(torch, dev):
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+        return vis.split(",")[dev] if vis else str(dev)
+
+
+def _algorithmic_bytes(w: wl.Workload):
+    """HBM bytes each kernel must move per launch, and L2 bytes of the array."""
+    nnz, nb, row = w.nnz, w.T * w.B, w.B * w.T * w.d * 4
+    stream = 8 * nnz + 8 * (nb + 1)
+    return {
+        "forward": stream + row,             # indices + offsets read, out written
+        "scatter": stream + row,             # indices + offsets read, grad_out read
+        "l2_gather": 4 * nnz * w.d,          # hashed blocks read from the shared array
+        "l2_scatter": 4 * nnz * w.d,         # vector atomics into the shared array
+    }
+
+
+def _oracle_sample(w: wl.Workload, rows: int):
+    """First ``rows`` batch rows of every table as a smaller batch."""
+    idx_parts, lens = [], []
+    for t in range(w.T):
+        for b in range(rows):
+            s = t * w.B + b
+            idx_parts.append(w.indices[w.offsets[s]:w.offsets[s + 1]])
+            lens.append(idx_parts[-1].shape[0])
+    off = np.zeros(len(lens) + 1, dtype=np.int64)
+    np.cumsum(lens, out=off[1:])
+    go = w.grad_out.reshape(w.B, w.T, w.d)[:rows].reshape(-1).copy()
+    return np.concatenate(idx_parts).astype(np.int64), off, go
+
+
+def _oracle_rate(w: wl.Workload, budget_s: float, max_rows: int = None):
+    """Time the CPU oracle (as it stands) on bounded samples of the workload."""
+    import oracle
+    o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed)
+    wcur = w.w0.copy() if w.w0 is not None else None
+    Gcur = np.zeros(w.M, np.float32)
+    rows = min(w.B, max_rows or 256)
+    # grow the sample until one step takes about budget/5
+    while True:
+        idx, off, go = _oracle_sample(w, rows)
+        t0 = time.perf_counter()
+        out, _ = o.forward(wcur, idx, off, rows)
+        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+        dt = time.perf_counter() - t0
+        if dt > budget_s / 5 or rows >= w.B or (max_rows and rows >= max_rows):
+            break
+        rows = min(w.B, rows * 2)
+    reps, tot, lookups = 0, 0.0, 0
+    while tot < budget_s and reps < 20:
+        t0 = time.perf_counter()
+        out, _ = o.forward(wcur, idx, off, rows)
+        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+        tot += time.perf_counter() - t0
+        reps += 1
+        lookups += idx.shape[0]
+    return lookups / tot, rows, reps, idx.shape[0], tot
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle timed on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    w = wl.make_workload(args.workload, M=args.M)
+    import oracle
+    o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed)
+    total_budget = 90.0
+    per_step = total_budget / max(1, args.steps + args.warmup)
+    # size the per-step sample so K+W steps fit the budget
+    rows = 64
+    idx, off, go = _oracle_sample(w, rows)
+    t0 = time.perf_counter()
+    wcur, Gcur = w.w0.copy(), np.zeros(w.M, np.float32)
+    o.forward(wcur, idx, off, rows)
+    o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+    dt = time.perf_counter() - t0
+    rows = int(max(1, min(w.B, rows * per_step / max(dt, 1e-6) * 0.8)))
+    idx, off, go = _oracle_sample(w, rows)
+    for _ in range(args.warmup):
+        o.forward(wcur, idx, off, rows)
+        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        o.forward(wcur, idx, off, rows)
+        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+    el = time.perf_counter() - t0
+    value = idx.shape[0] * args.steps / el
+    sample = (f"first {rows} of {w.B} batch rows x {w.T} tables ({idx.shape[0]} lookups) per step; "
+              "forward + gradient + update, single thread")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64+f32",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B, "seq_len": 1,
+                   "parallelism": "single host thread"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2207_10731_gb300 import binding
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != args.gpus:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE={world}")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    # one replica per rank, each with its own batch (no data-path exchange)
+    w = wl.make_workload(args.workload, seed=0, M=args.M)
+    batches = [(w.indices, w.offsets, w.grad_out)]
+    for k in range(1, args.rotate):
+        batches.append(wl.make_batch(w.cards, w.B, w.d, wl.CONFIGS[args.workload]["bag"],
+                                     wl.CONFIGS[args.workload]["ids"], seed=rank, batch=k,
+                                     grad=wl.CONFIGS[args.workload].get("grad", "normal")))
+    dbatches = [(torch.from_numpy(i).to(dev), torch.from_numpy(o).to(dev),
+                 torch.from_numpy(g).to(dev)) for i, o, g in batches]
+    h = binding.PSS(w.cards, dim=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, optimizer=w.opt,
+                    eps=w.eps)
+    if w.w0 is not None:
+        h.set_weights(torch.from_numpy(w.w0).to(dev))
+    else:
+        base = torch.from_numpy(w.w0_base).to(dev)
+        h.set_weights(base.repeat(-(-w.M // base.numel()))[: w.M].contiguous())
+        del base
+    out = torch.empty((w.B, w.T, w.d), dtype=torch.float32, device=dev)
+    nnz_per_step = [int(b[0].shape[0]) for b in batches]
+    stream = torch.cuda.current_stream()
+
+    def step(k):
+        i, o, g = dbatches[k % len(dbatches)]
+        h.forward(i, o, w.B, out=out)
+        h.backward_update(g, w.lr)
+
+    for k in range(args.warmup):
+        step(k)
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(_gpu_id(torch, local)) if rank == 0 else None
+    time.sleep(0.3 if sampler else 0)
+    h.set_option(binding.OPT_PROFILE, 1)
+    h.reset_profile()
+    launches0 = h.info()["kernel_launches"]
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    wall0 = time.time()
+    ev0.record(stream)
+    for k in range(args.steps):
+        step(k)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    wall1 = time.time()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    launches = h.info()["kernel_launches"] - launches0
+    prof = {}
+    for kid, name in enumerate(binding.KERNEL_NAMES):
+        n, ms = h.profile(kid)
+        if n:
+            prof[name] = (n, ms)
+    h.set_option(binding.OPT_PROFILE, 0)
+    if sampler:
+        time.sleep(0.3)
+        sampler.stop()
+    lookups = sum(nnz_per_step[k % len(nnz_per_step)] for k in range(args.steps))
+    if world > 1:
+        t = torch.tensor([elapsed_ms, float(lookups)], dtype=torch.float64, device=dev)
+        tmax = t.clone()
+        dist.all_reduce(tmax[:1], op=dist.ReduceOp.MAX)
+        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
+        elapsed_ms, lookups = float(tmax[0]), float(t[1])
+
+    # end to end through the same C-ABI calls with pinned HOST buffers:
+    # every step copies indices, offsets and grad_out in and the pooled output out.
+    e2e_steps = max(3, min(args.steps, args.e2e_steps))
+    hb = [(torch.from_numpy(i).pin_memory(), torch.from_numpy(o).pin_memory(),
+           torch.from_numpy(g).pin_memory()) for i, o, g in batches]
+    hout = torch.empty((w.B, w.T, w.d), dtype=torch.float32, pin_memory=True)
+
+    def step_host(k):
+        i, o, g = hb[k % len(hb)]
+        h.forward(i, o, w.B, out=hout)
+        h.backward_update(g, w.lr)
+
+    step_host(0)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for k in range(e2e_steps):
+        step_host(k)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    e2e_lookups = sum(nnz_per_step[k % len(nnz_per_step)] for k in range(e2e_steps))
+    if world > 1:
+        t = torch.tensor([e2e_ms, float(e2e_lookups)], dtype=torch.float64, device=dev)
+        tmax = t.clone()
+        dist.all_reduce(tmax[:1], op=dist.ReduceOp.MAX)
+        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
+        e2e_ms, e2e_lookups = float(tmax[0]), float(t[1])
+    h2d = int(np.mean([i.nbytes + o.nbytes + g.nbytes for i, o, g in batches]))
+    d2h = int(hout.numel() * 4)
+
+    if rank == 0:
+        clocks = sampler.summary(wall0, wall1) if sampler else None
+        value = lookups / (elapsed_ms / 1e3)
+        peak, peak_kind = _peaks()
+        ab = _algorithmic_bytes(w)
+        dom = max(prof.items(), key=lambda kv: kv[1][1])[0] if prof else "forward"
+        n_dom, ms_dom = prof.get(dom, (1, float("nan")))
+        avg_s = ms_dom / max(1, n_dom) / 1e3
+        bytes_dom = ab.get(dom, ab["forward"])
+        achieved = bytes_dom / avg_s / 1e9
+        step_bytes = ab["forward"] + ab["scatter"]
+        step_gbs = step_bytes / (elapsed_ms / args.steps / 1e3) / 1e9 * world
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            rate, rows, reps, nnz_s, tot = _oracle_rate(w, args.cpu_budget)
+            cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
+                   "sample": (f"first {rows} of {w.B} batch rows x {w.T} tables "
+                              f"({nnz_s} lookups) per step, {reps} steps, {tot:.1f} s: forward + "
+                              "gradient + update, single host thread")}
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B * world,
+                       "seq_len": 1,
+                       "parallelism": "independent replicas" if world > 1 else "single GPU",
+                       "l2": (f"inputs larger than L2: {args.rotate}-batch rotation, "
+                              f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB output and "
+                              f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB upstream gradient per step")},
+            "step_gbs": step_gbs,
+            "bags_per_s": w.B * w.T * args.steps * world / (elapsed_ms / 1e3),
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
+                         "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": _traffic(dom, args.workload),
+                         "peak_kind": peak_kind, "algorithmic_bytes_per_launch": bytes_dom,
+                         "avg_launch_ms": avg_s * 1e3,
+                         "step_frac": step_gbs / world / peak},
+            "kernels_ms": {k: v[1] / v[0] for k, v in prof.items()},
+            "gpu_launches": launches * world,
+            "e2e": {"value": e2e_lookups / (e2e_ms / 1e3), "unit": UNIT,
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "steps": e2e_steps},
+            "cpu_baseline": cpu,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    h.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(wl.CONFIGS), default="tb")
+    ap.add_argument("--M", type=int, default=None, help="shared-array length (sweep workload)")
+    ap.add_argument("--rotate", type=int, default=2, help="distinct batches cycled through")
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle timing")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be at least 3")
+    if args.workload == "sweep" and args.M is None:
+        args.M = 1 << 24
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

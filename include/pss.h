@@ -1,0 +1,228 @@
+/*
+ * pss.h -- C ABI of libpss.so: the hashed shared-array embedding ("parameter
+ * sharing setup", PSS, with the ROBE-Z mapping) of Desai & Shrivastava, "The
+ * trade-offs of model size in large recommendation models" (arXiv 2207.10731),
+ * on one NVIDIA GB300 (sm_103a).
+ *
+ * The method (Def. 1, Sec. 2.1; Sec. 2.4; ROBE-Z mapping of Sec. 2.5):
+ *   All T embedding tables share ONE learnable fp32 array M of length `M`.
+ *   Chunk j (0 <= j < J, J = ceil(d/Z)) of the embedding of id i of table t is
+ *   the contiguous block  M[loc(t,i,j) : loc(t,i,j) + L_j],  L_j = min(Z, d - jZ).
+ *   A bag's output is the sum of the embeddings of its ids (sum pooling), so
+ *       out[b][t][jZ + z] = sum over ids i of bag (t,b) of  M[loc(t,i,j) + z].
+ *   The backward pass adds each bag's upstream gradient back into every block
+ *   it read (the dense branch of Algorithm 1, Sec. 3), and the optimizer step
+ *   (SGD or Adagrad) is applied to M in the same call.
+ *
+ * The location hash (Sec. 2.5 asks only for a universal hash; the choices below
+ * are this library's, fixed so that results are reproducible bit for bit):
+ *   P   = 2^61 - 1 (Mersenne prime)
+ *   A   = 1 + (s1 mod (P-1)),  B0 = s2 mod P, where s1, s2 are the first two
+ *         outputs of splitmix64 (Steele, Lea & Flood 2014) seeded with `seed`
+ *   key = ((i*T + t)*J + j)                          (unsigned 64-bit)
+ *   x   = (A*key + B0) mod P                         (exact, 128-bit product)
+ *   L   = min(Z, d),   R = floor((M - L)/G) + 1
+ *   loc = G * (x mod R)                              (so 0 <= loc <= M - L)
+ *   G ("alignment") is the granularity of block starts: G = 4 makes every
+ *   block 16-byte aligned; G = 1 is the paper's arbitrary offset.
+ *
+ * Batch layout (all int64, CSR, TABLE-MAJOR bags):
+ *   bag (t, b) is slot s = t*B + b and owns indices[offsets[s] .. offsets[s+1]);
+ *   offsets has T*B + 1 entries, non-decreasing, offsets[0] >= 0,
+ *   offsets[T*B] <= nnz.  Pooled outputs and upstream gradients are fp32,
+ *   row-major [B][T][d] (the DLRM concatenation order).
+ *
+ * Memory and streams:
+ *   The library owns M, the Adagrad accumulator, its gradient scratch and all
+ *   staging buffers; the caller owns every pointer it passes.  Calls taking a
+ *   `stream` are asynchronous on it (stream-ordered) unless stated otherwise;
+ *   the caller's buffers must stay valid until that work completes.  Batch
+ *   pointers may be device memory or host memory (pinned or pageable): host
+ *   batches are staged through library-owned device buffers on the same
+ *   stream.  A handle is not thread-safe; use one handle per thread or lock.
+ *
+ * Errors: every call returns a pss_status; none aborts the process.  Bad
+ * arguments are rejected on the host before any work is queued.  An id outside
+ * [0, n_t) cannot be seen on the host; the device skips that id (it contributes
+ * nothing) and records the smallest such position in a device error word,
+ * which pss_get_error() reads and clears.
+ */
+#ifndef PSS_H_
+#define PSS_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pss_handle pss_handle;
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* pss_stream;
+
+typedef enum {
+    PSS_OK = 0,
+    PSS_ERR_INVALID_ARG = 1,   /* a size, pointer or option value is invalid */
+    PSS_ERR_OOM = 2,           /* a device allocation failed */
+    PSS_ERR_CUDA = 3,          /* a CUDA runtime call failed */
+    PSS_ERR_STATE = 4,         /* call order violated (e.g. backward before forward) */
+    PSS_ERR_INDEX_RANGE = 5,   /* the device saw an id outside its table, or bad offsets */
+    PSS_ERR_TIMEOUT = 6,       /* a bounded device wait gave up */
+    PSS_ERR_UNSUPPORTED = 7    /* valid request this build does not implement */
+} pss_status;
+
+typedef enum { PSS_SGD = 0, PSS_ADAGRAD = 1 } pss_optimizer;
+
+/* Option keys for pss_set_option / pss_get_option. */
+typedef enum {
+    /* Backward path: the dense gradient of Algorithm 1 built with vector atomics
+     * (PSS_PATH_ATOMIC), or the sorted, deterministic path that reduces equal
+     * locations before touching M (PSS_PATH_SORTED, Algorithm 1's sparse branch).
+     * PSS_PATH_AUTO picks by the measured collision rate of the previous batch. */
+    PSS_OPT_BACKWARD_PATH = 1,
+    /* How the Adagrad step visits M: every element (PSS_UPDATE_DENSE), only the
+     * blocks the batch touched (PSS_UPDATE_TOUCHED), or chosen from M and the
+     * batch size (PSS_UPDATE_AUTO).  Results are identical. */
+    PSS_OPT_UPDATE_MODE = 2,
+    /* 1: record CUDA events around every kernel (read with pss_get_profile). */
+    PSS_OPT_PROFILE = 3,
+    /* 1: forward/backward synchronise the stream and return
+     * PSS_ERR_INDEX_RANGE at once when the device error word is set. */
+    PSS_OPT_SYNC_CHECK = 4
+} pss_option;
+
+enum { PSS_PATH_AUTO = 0, PSS_PATH_ATOMIC = 1, PSS_PATH_SORTED = 2 };
+enum { PSS_UPDATE_AUTO = 0, PSS_UPDATE_DENSE = 1, PSS_UPDATE_TOUCHED = 2 };
+
+/* Kernel ids for pss_get_profile. */
+typedef enum {
+    PSS_K_LOCATIONS = 0,   /* hash only (pss_compute_locations) */
+    PSS_K_FORWARD = 1,     /* fused hash + gather + sum-pool */
+    PSS_K_SCATTER = 2,     /* backward: hash + vector-atomic scatter (+ fused SGD) */
+    PSS_K_UPDATE = 3,      /* optimizer pass over M (dense or touched blocks) */
+    PSS_K_SORT = 4,        /* sorted path: key build + radix sort passes */
+    PSS_K_REDUCE = 5,      /* sorted path: segmented reduce + fused update */
+    PSS_K_MISC = 6,        /* memsets and small helper kernels */
+    PSS_K_COUNT = 7
+} pss_kernel_id;
+
+/* Read-only description of a handle. */
+typedef struct {
+    int64_t T, d, M, Z, G, J, L, R;
+    uint64_t A, B0;            /* hash parameters derived from the seed */
+    int64_t optimizer;         /* pss_optimizer */
+    int64_t kernel_launches;   /* kernels this handle has launched so far */
+    int64_t last_path;         /* PSS_PATH_ATOMIC / PSS_PATH_SORTED of the last backward */
+    double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass, or -1 */
+} pss_info;
+
+/*
+ * Create a PSS instance (Def. 1, Sec. 2.1; ROBE-Z mapping, Sec. 2.5).
+ *   table_cardinalities: host, num_tables entries n_t >= 1 (ids of table t are
+ *                        0 .. n_t - 1).  Copied; the caller keeps ownership.
+ *   dim (d):  1 .. 512.   Z: chunk length >= 1.   G: block-start alignment >= 1.
+ *   M:        shared-array length in fp32 elements, M >= min(Z, d); 64-bit.
+ *   seed:     hash seed (see the header comment).
+ *   opt:      PSS_SGD or PSS_ADAGRAD;  adagrad_eps: Adagrad epsilon (> 0).
+ * M (and, for Adagrad, the accumulator) is allocated on the current device and
+ * zero-filled on `stream`; load initial values with pss_set_weights.
+ * Errors: PSS_ERR_INVALID_ARG (sizes, null pointers, max_t n_t * T * J > 2^61-1),
+ * PSS_ERR_OOM, PSS_ERR_CUDA.  *out is set only on success.
+ */
+pss_status pss_create(const int64_t* table_cardinalities, int32_t num_tables, int32_t dim,
+                      int64_t M, int32_t Z, int32_t G, uint64_t seed, pss_optimizer opt,
+                      float adagrad_eps, pss_stream stream, pss_handle** out);
+
+/* Free every device buffer of the handle (synchronises the device first). NULL is a no-op. */
+pss_status pss_destroy(pss_handle* h);
+
+/* Copy n == M fp32 values into the shared array.  `w` is host or device memory.
+ * Errors: PSS_ERR_INVALID_ARG (NULL, n != M), PSS_ERR_CUDA. */
+pss_status pss_set_weights(pss_handle* h, const float* w, int64_t n, pss_stream stream);
+
+/* Copy the shared array out (n == M).  Stream-ordered: synchronise `stream`
+ * before reading a host buffer. */
+pss_status pss_get_weights(pss_handle* h, float* w, int64_t n, pss_stream stream);
+
+/* Checkpoint: copy M and the Adagrad accumulator (n == M each) to / from the
+ * caller.  `G` is ignored (may be NULL) for SGD.  Host or device pointers. */
+pss_status pss_get_state(pss_handle* h, float* w, float* G, int64_t n, pss_stream stream);
+pss_status pss_set_state(pss_handle* h, const float* w, const float* G, int64_t n,
+                         pss_stream stream);
+
+/*
+ * The mapping matrix of Algorithm 1 ("locations from which the output was
+ * accessed"): locs[q*J + j] = loc(t, indices[q], j) for every id position q of
+ * every bag, as an element offset into M; -1 for an id outside [0, n_t)
+ * (that position is also recorded in the error word).  Positions not covered
+ * by any bag are left untouched.
+ *   indices: int64[nnz], offsets: int64[T*B+1] (table-major), B >= 0,
+ *   locs:    int64[nnz*J].  Device or host pointers.
+ */
+pss_status pss_compute_locations(pss_handle* h, const int64_t* indices, int64_t nnz,
+                                 const int64_t* offsets, int64_t B, int64_t* locs,
+                                 pss_stream stream);
+
+/*
+ * Forward pass (Sec. 2.4 forward(i) = (S e_i)^T M, sum-pooled per bag):
+ *   out[b][t][k] = sum over q in bag (t,b) of M[loc(t, indices[q], k / Z) + k % Z].
+ * An empty bag gives a zero row.  out: fp32[B*T*d], fully overwritten.
+ * The batch (indices, offsets, nnz, B) is remembered by pointer for the next
+ * pss_backward_update / pss_backward_grad: the caller must keep it unchanged
+ * until that call's work has completed.  Host batches are staged (and `out`
+ * copied back) on `stream`.
+ */
+pss_status pss_forward(pss_handle* h, const int64_t* indices, int64_t nnz,
+                       const int64_t* offsets, int64_t B, float* out, pss_stream stream);
+
+/*
+ * Backward pass fused with the optimizer step for the batch of the last
+ * pss_forward (Sec. 2.4 backward(i, D) = (S e_i) D; Algorithm 1; SGD / Adagrad):
+ *   g[e] = sum over every (bag, id, chunk j, z) with loc + z == e of grad_out[b][t][jZ+z]
+ *   SGD:     M[e] -= lr * g[e]
+ *   Adagrad: G[e] += g[e]^2;  M[e] -= lr * g[e] / (sqrt(G[e]) + eps)   (only where g[e] != 0)
+ * grad_out: fp32[B*T*d] (device or host).  lr: any finite value (lr = 0 leaves
+ * M unchanged).  Errors: PSS_ERR_STATE if no forward has been run.
+ */
+pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, pss_stream stream);
+
+/*
+ * Gradient only (Algorithm 1, dense branch output G_i): writes g (above) for
+ * the batch of the last pss_forward into grad (fp32[M], DEVICE memory),
+ * overwriting it; M and the optimizer state are not changed.
+ */
+pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, pss_stream stream);
+
+/* Set / get an option (pss_option).  Invalid key or value: PSS_ERR_INVALID_ARG. */
+pss_status pss_set_option(pss_handle* h, int32_t key, int64_t value);
+pss_status pss_get_option(pss_handle* h, int32_t key, int64_t* value);
+
+/*
+ * Synchronise `stream`, then read and clear the device error word.
+ * *first_bad_index = smallest id position q seen outside its table since the
+ * last call, or -1.  Returns PSS_ERR_INDEX_RANGE if an id or the offsets were
+ * bad (offsets problems set *first_bad_index to -2 when no id was bad),
+ * PSS_OK otherwise.
+ */
+pss_status pss_get_error(pss_handle* h, int64_t* first_bad_index, pss_stream stream);
+
+/* Fill *info (host). */
+pss_status pss_get_info(pss_handle* h, pss_info* info);
+
+/*
+ * Profiling (with PSS_OPT_PROFILE = 1): synchronise, then report for kernel id
+ * `kernel` the number of launches and their summed device time in ms since the
+ * last pss_reset_profile.  Times come from CUDA events recorded on the launch
+ * stream immediately around each launch.
+ */
+pss_status pss_get_profile(pss_handle* h, int32_t kernel, int64_t* launches, double* total_ms);
+pss_status pss_reset_profile(pss_handle* h);
+
+/* Static description of a status code. */
+const char* pss_status_string(pss_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PSS_H_ */

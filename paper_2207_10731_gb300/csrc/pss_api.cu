@@ -1,0 +1,615 @@
+// C ABI of libpss.so (declared in include/pss.h): handle life cycle, argument
+// validation, staging of host batches, backward-path dispatch and profiling.
+#include <climits>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "pss.h"
+#include "pss_internal.h"
+
+using namespace pss;
+
+namespace {
+
+// Restores the caller's current device on scope exit.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = false;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) == cudaSuccess) ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+struct Staging {
+    void* ptr = nullptr;
+    size_t cap = 0;
+};
+
+struct EventPair {
+    cudaEvent_t a, b;
+};
+
+}  // namespace
+
+struct pss_handle {
+    int device = 0;
+    int sm_count = 0;
+    DevParams dp{};
+    RowLayout layout{};
+    std::vector<int64_t> cards;
+    pss_optimizer opt = PSS_SGD;
+    float eps = 1e-10f;
+
+    float* w = nullptr;          // shared array M (library-owned)
+    float* Gacc = nullptr;       // Adagrad accumulator
+    float* g = nullptr;          // dense gradient scratch, zero between calls
+    int64_t* cards_dev = nullptr;
+    DevError* err = nullptr;
+
+    // batch of the last forward (device pointers: the caller's or staged)
+    const int64_t* last_idx = nullptr;
+    const int64_t* last_off = nullptr;
+    int64_t last_nnz = 0, last_B = 0;
+    bool have_batch = false;
+
+    // options
+    int64_t path = PSS_PATH_AUTO;
+    int64_t update_mode = PSS_UPDATE_AUTO;
+    int64_t profile = 0;
+    int64_t sync_check = 0;
+    int64_t last_path = PSS_PATH_ATOMIC;
+    double last_collision = -1.0;
+
+    Staging st_idx, st_off, st_out, st_grad, st_locs;
+
+    // touched-block bookkeeping (allocated on first use)
+    Touched touched{};
+    int64_t touched_words = 0;
+
+    // profiling
+    std::vector<EventPair> ev[PSS_K_COUNT];
+    std::vector<EventPair> ev_free;
+    int64_t launches_by_kernel[PSS_K_COUNT] = {0};
+    int64_t launches = 0;
+};
+
+namespace {
+
+pss_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return PSS_OK;
+    if (e == cudaErrorMemoryAllocation) return PSS_ERR_OOM;
+    return PSS_ERR_CUDA;
+}
+
+#define PSS_TRY(expr)                                  \
+    do {                                               \
+        pss_status _s = cuda_status(expr);             \
+        if (_s != PSS_OK) return _s;                   \
+    } while (0)
+
+bool is_device_ptr(const void* p) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+cudaError_t ensure(Staging& s, size_t bytes, cudaStream_t st) {
+    if (bytes == 0) bytes = 16;
+    if (s.cap >= bytes) return cudaSuccess;
+    if (s.ptr) {
+        cudaError_t e = cudaFreeAsync(s.ptr, st);
+        if (e != cudaSuccess) return e;
+        s.ptr = nullptr;
+        s.cap = 0;
+    }
+    cudaError_t e = cudaMallocAsync(&s.ptr, bytes, st);
+    if (e == cudaSuccess) s.cap = bytes;
+    return e;
+}
+
+// Device view of a caller buffer: the pointer itself, or a staged copy.
+template <typename T>
+pss_status device_view(const T* p, size_t count, Staging& s, cudaStream_t st, const T** out) {
+    if (count == 0 || is_device_ptr(p)) {
+        *out = p;
+        return PSS_OK;
+    }
+    PSS_TRY(ensure(s, count * sizeof(T), st));
+    PSS_TRY(cudaMemcpyAsync(s.ptr, p, count * sizeof(T), cudaMemcpyHostToDevice, st));
+    *out = static_cast<const T*>(s.ptr);
+    return PSS_OK;
+}
+
+EventPair take_events(pss_handle* h) {
+    if (!h->ev_free.empty()) {
+        EventPair e = h->ev_free.back();
+        h->ev_free.pop_back();
+        return e;
+    }
+    EventPair e{nullptr, nullptr};
+    cudaEventCreate(&e.a);
+    cudaEventCreate(&e.b);
+    return e;
+}
+
+// Bracket one launch: counts it and, when profiling, records events on its stream.
+struct LaunchScope {
+    pss_handle* h;
+    int k;
+    cudaStream_t st;
+    EventPair ev{nullptr, nullptr};
+    LaunchScope(pss_handle* h_, int k_, cudaStream_t st_) : h(h_), k(k_), st(st_) {
+        if (h->profile) {
+            ev = take_events(h);
+            cudaEventRecord(ev.a, st);
+        }
+    }
+    ~LaunchScope() {
+        h->launches++;
+        h->launches_by_kernel[k]++;
+        if (h->profile && ev.a) {
+            cudaEventRecord(ev.b, st);
+            h->ev[k].push_back(ev);
+        }
+    }
+};
+
+pss_status check_error_word(pss_handle* h, cudaStream_t st, int64_t* first_bad) {
+    DevError e;
+    PSS_TRY(cudaMemcpyAsync(&e, h->err, sizeof(e), cudaMemcpyDeviceToHost, st));
+    PSS_TRY(cudaStreamSynchronize(st));
+    DevError clear{ULLONG_MAX, 0u, 0u};
+    PSS_TRY(cudaMemcpyAsync(h->err, &clear, sizeof(clear), cudaMemcpyHostToDevice, st));
+    PSS_TRY(cudaStreamSynchronize(st));
+    int64_t fb = (e.first_bad == ULLONG_MAX) ? -1 : (int64_t)e.first_bad;
+    if (fb < 0 && (e.flags & kErrOffsets)) fb = -2;
+    if (first_bad) *first_bad = fb;
+    return (fb != -1) ? PSS_ERR_INDEX_RANGE : PSS_OK;
+}
+
+pss_status ensure_grad(pss_handle* h, cudaStream_t st) {
+    if (h->g) return PSS_OK;
+    PSS_TRY(cudaMalloc(&h->g, sizeof(float) * (size_t)h->dp.M));
+    PSS_TRY(cudaMemsetAsync(h->g, 0, sizeof(float) * (size_t)h->dp.M, st));
+    return PSS_OK;
+}
+
+pss_status ensure_touched(pss_handle* h, int64_t pairs, cudaStream_t st) {
+    const int64_t R = (int64_t)h->dp.R;
+    int64_t need = pairs < R ? pairs : R;
+    if (need < 1) need = 1;
+    if (!h->touched.bitmap) {
+        const int64_t extra = (int64_t)h->dp.L / h->dp.G + 64;
+        h->touched_words = (R + extra) / 32 + 2;
+        PSS_TRY(cudaMalloc(&h->touched.bitmap, sizeof(uint32_t) * (size_t)h->touched_words));
+        PSS_TRY(cudaMemsetAsync(h->touched.bitmap, 0, sizeof(uint32_t) * (size_t)h->touched_words, st));
+        PSS_TRY(cudaMalloc(&h->touched.count, sizeof(unsigned long long)));
+        PSS_TRY(cudaMemsetAsync(h->touched.count, 0, sizeof(unsigned long long), st));
+    }
+    if (h->touched.cap < need) {
+        if (h->touched.list) PSS_TRY(cudaFreeAsync(h->touched.list, st));
+        h->touched.list = nullptr;
+        h->touched.cap = 0;
+        PSS_TRY(cudaMallocAsync(&h->touched.list, sizeof(int64_t) * (size_t)need, st));
+        h->touched.cap = need;
+    }
+    return PSS_OK;
+}
+
+bool use_touched(const pss_handle* h, int64_t pairs) {
+    if (h->update_mode == PSS_UPDATE_DENSE) return false;
+    if (h->update_mode == PSS_UPDATE_TOUCHED) return true;
+    // dense pass reads/writes ~5 words per element of M; the touched pass
+    // costs ~5 words per element of each distinct block plus the marking.
+    return h->dp.M > 2 * pairs * (int64_t)h->dp.L;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+RowLayout layout_for(const pss_handle* h, const void* rowbuf) {
+    if (h->layout.vw == 4 && !aligned16(rowbuf)) return choose_layout(h->dp.d, 1, 1);
+    return h->layout;
+}
+
+pss_status validate_batch(const pss_handle* h, const int64_t* idx, int64_t nnz,
+                          const int64_t* off, int64_t B) {
+    if (!off || B < 0 || nnz < 0 || (nnz > 0 && !idx)) return PSS_ERR_INVALID_ARG;
+    if (B > (INT64_MAX / 2) / h->dp.T) return PSS_ERR_INVALID_ARG;
+    return PSS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* pss_status_string(pss_status s) {
+    switch (s) {
+        case PSS_OK: return "ok";
+        case PSS_ERR_INVALID_ARG: return "invalid argument";
+        case PSS_ERR_OOM: return "device out of memory";
+        case PSS_ERR_CUDA: return "CUDA runtime error";
+        case PSS_ERR_STATE: return "invalid call order";
+        case PSS_ERR_INDEX_RANGE: return "id outside its table, or malformed offsets";
+        case PSS_ERR_TIMEOUT: return "device wait timed out";
+        case PSS_ERR_UNSUPPORTED: return "unsupported";
+    }
+    return "unknown status";
+}
+
+pss_status pss_create(const int64_t* cards, int32_t T, int32_t dim, int64_t M, int32_t Z,
+                      int32_t G, uint64_t seed, pss_optimizer opt, float adagrad_eps,
+                      pss_stream stream, pss_handle** out) {
+    if (!out || !cards || T <= 0 || dim <= 0 || dim > 512 || Z <= 0 || G <= 0 || M <= 0)
+        return PSS_ERR_INVALID_ARG;
+    if (opt != PSS_SGD && opt != PSS_ADAGRAD) return PSS_ERR_INVALID_ARG;
+    if (opt == PSS_ADAGRAD && !(adagrad_eps > 0.f)) return PSS_ERR_INVALID_ARG;
+    const int64_t J = (dim + Z - 1) / Z;
+    const int64_t L = Z < dim ? Z : dim;
+    if (M < L) return PSS_ERR_INVALID_ARG;
+    int64_t max_card = 0;
+    for (int32_t t = 0; t < T; ++t) {
+        if (cards[t] <= 0) return PSS_ERR_INVALID_ARG;
+        if (cards[t] > max_card) max_card = cards[t];
+    }
+    const unsigned __int128 P = (((unsigned __int128)1) << 61) - 1;
+    if ((unsigned __int128)max_card * (unsigned __int128)T * (unsigned __int128)J > P)
+        return PSS_ERR_INVALID_ARG;
+
+    pss_handle* h = new (std::nothrow) pss_handle();
+    if (!h) return PSS_ERR_OOM;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaGetDevice(&h->device) != cudaSuccess) {
+        delete h;
+        return PSS_ERR_CUDA;
+    }
+    cudaDeviceGetAttribute(&h->sm_count, cudaDevAttrMultiProcessorCount, h->device);
+    if (h->sm_count <= 0) h->sm_count = 1;
+
+    // hash parameters from splitmix64(seed)
+    uint64_t s = seed;
+    auto next = [&s]() {
+        s += 0x9e3779b97f4a7c15ULL;
+        uint64_t z = s;
+        z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ULL;
+        z = (z ^ (z >> 27)) * 0x94d049bb133111ebULL;
+        return z ^ (z >> 31);
+    };
+    const uint64_t p61 = (uint64_t(1) << 61) - 1;
+    const uint64_t s1 = next(), s2 = next();
+    DevParams& dp = h->dp;
+    dp.A = 1 + s1 % (p61 - 1);
+    dp.B0 = s2 % p61;
+    dp.G = G;
+    dp.M = M;
+    dp.T = T;
+    dp.d = dim;
+    dp.Z = Z;
+    dp.J = (int32_t)J;
+    dp.L = (int32_t)L;
+    dp.R = (uint64_t)((M - L) / G + 1);
+    dp.Rinv = UINT64_MAX / dp.R;
+    h->layout = choose_layout(dim, Z, G);
+    h->cards.assign(cards, cards + T);
+    h->opt = opt;
+    h->eps = adagrad_eps;
+
+    pss_status rc = PSS_OK;
+    do {
+        if ((rc = cuda_status(cudaMalloc(&h->w, sizeof(float) * (size_t)M))) != PSS_OK) break;
+        if ((rc = cuda_status(cudaMemsetAsync(h->w, 0, sizeof(float) * (size_t)M, st))) != PSS_OK) break;
+        if (opt == PSS_ADAGRAD) {
+            if ((rc = cuda_status(cudaMalloc(&h->Gacc, sizeof(float) * (size_t)M))) != PSS_OK) break;
+            if ((rc = cuda_status(cudaMemsetAsync(h->Gacc, 0, sizeof(float) * (size_t)M, st))) != PSS_OK) break;
+            if ((rc = ensure_grad(h, st)) != PSS_OK) break;
+        }
+        if ((rc = cuda_status(cudaMalloc(&h->cards_dev, sizeof(int64_t) * (size_t)T))) != PSS_OK) break;
+        if ((rc = cuda_status(cudaMemcpy(h->cards_dev, cards, sizeof(int64_t) * (size_t)T,
+                                         cudaMemcpyHostToDevice))) != PSS_OK) break;
+        if ((rc = cuda_status(cudaMalloc(&h->err, sizeof(DevError)))) != PSS_OK) break;
+        DevError clear{ULLONG_MAX, 0u, 0u};
+        if ((rc = cuda_status(cudaMemcpy(h->err, &clear, sizeof(clear), cudaMemcpyHostToDevice))) != PSS_OK) break;
+        if ((rc = cuda_status(cudaStreamSynchronize(st))) != PSS_OK) break;
+    } while (0);
+    dp.cards = h->cards_dev;
+    if (rc != PSS_OK) {
+        pss_destroy(h);
+        return rc;
+    }
+    *out = h;
+    return PSS_OK;
+}
+
+pss_status pss_destroy(pss_handle* h) {
+    if (!h) return PSS_OK;
+    DeviceGuard g(h->device);
+    cudaDeviceSynchronize();
+    cudaFree(h->w);
+    cudaFree(h->Gacc);
+    cudaFree(h->g);
+    cudaFree(h->cards_dev);
+    cudaFree(h->err);
+    cudaFree(h->touched.bitmap);
+    cudaFree(h->touched.list);
+    cudaFree(h->touched.count);
+    for (Staging* s : {&h->st_idx, &h->st_off, &h->st_out, &h->st_grad, &h->st_locs})
+        if (s->ptr) cudaFree(s->ptr);
+    for (int k = 0; k < PSS_K_COUNT; ++k)
+        for (auto& e : h->ev[k]) {
+            cudaEventDestroy(e.a);
+            cudaEventDestroy(e.b);
+        }
+    for (auto& e : h->ev_free) {
+        cudaEventDestroy(e.a);
+        cudaEventDestroy(e.b);
+    }
+    delete h;
+    return PSS_OK;
+}
+
+pss_status pss_set_weights(pss_handle* h, const float* w, int64_t n, pss_stream stream) {
+    if (!h || !w || n != h->dp.M) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    PSS_TRY(cudaMemcpyAsync(h->w, w, sizeof(float) * (size_t)n, cudaMemcpyDefault,
+                            reinterpret_cast<cudaStream_t>(stream)));
+    return PSS_OK;
+}
+
+pss_status pss_get_weights(pss_handle* h, float* w, int64_t n, pss_stream stream) {
+    if (!h || !w || n != h->dp.M) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    PSS_TRY(cudaMemcpyAsync(w, h->w, sizeof(float) * (size_t)n, cudaMemcpyDefault,
+                            reinterpret_cast<cudaStream_t>(stream)));
+    return PSS_OK;
+}
+
+pss_status pss_get_state(pss_handle* h, float* w, float* G, int64_t n, pss_stream stream) {
+    if (!h || !w || n != h->dp.M || (h->opt == PSS_ADAGRAD && !G)) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    PSS_TRY(cudaMemcpyAsync(w, h->w, sizeof(float) * (size_t)n, cudaMemcpyDefault, st));
+    if (h->opt == PSS_ADAGRAD)
+        PSS_TRY(cudaMemcpyAsync(G, h->Gacc, sizeof(float) * (size_t)n, cudaMemcpyDefault, st));
+    return PSS_OK;
+}
+
+pss_status pss_set_state(pss_handle* h, const float* w, const float* G, int64_t n,
+                         pss_stream stream) {
+    if (!h || !w || n != h->dp.M || (h->opt == PSS_ADAGRAD && !G)) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    PSS_TRY(cudaMemcpyAsync(h->w, w, sizeof(float) * (size_t)n, cudaMemcpyDefault, st));
+    if (h->opt == PSS_ADAGRAD)
+        PSS_TRY(cudaMemcpyAsync(h->Gacc, G, sizeof(float) * (size_t)n, cudaMemcpyDefault, st));
+    return PSS_OK;
+}
+
+pss_status pss_compute_locations(pss_handle* h, const int64_t* indices, int64_t nnz,
+                                 const int64_t* offsets, int64_t B, int64_t* locs,
+                                 pss_stream stream) {
+    if (!h) return PSS_ERR_INVALID_ARG;
+    pss_status rc = validate_batch(h, indices, nnz, offsets, B);
+    if (rc != PSS_OK) return rc;
+    if (nnz > 0 && !locs) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int64_t nbags = (int64_t)h->dp.T * B;
+    const int64_t *di = nullptr, *doff = nullptr;
+    if ((rc = device_view(indices, (size_t)nnz, h->st_idx, st, &di)) != PSS_OK) return rc;
+    if ((rc = device_view(offsets, (size_t)(nbags + 1), h->st_off, st, &doff)) != PSS_OK) return rc;
+    const size_t nloc = (size_t)nnz * (size_t)h->dp.J;
+    int64_t* dl = locs;
+    const bool host_out = nloc > 0 && !is_device_ptr(locs);
+    if (host_out) {
+        PSS_TRY(ensure(h->st_locs, nloc * sizeof(int64_t), st));
+        dl = static_cast<int64_t*>(h->st_locs.ptr);
+        PSS_TRY(cudaMemcpyAsync(dl, locs, nloc * sizeof(int64_t), cudaMemcpyHostToDevice, st));
+    }
+    if (nbags > 0) {
+        LaunchScope ls(h, PSS_K_LOCATIONS, st);
+        PSS_TRY(launch_locations(h->dp, di, nnz, doff, B, dl, h->err, h->sm_count, st));
+    }
+    if (host_out)
+        PSS_TRY(cudaMemcpyAsync(locs, dl, nloc * sizeof(int64_t), cudaMemcpyDeviceToHost, st));
+    if (h->sync_check) return check_error_word(h, st, nullptr);
+    return PSS_OK;
+}
+
+pss_status pss_forward(pss_handle* h, const int64_t* indices, int64_t nnz, const int64_t* offsets,
+                       int64_t B, float* out, pss_stream stream) {
+    if (!h) return PSS_ERR_INVALID_ARG;
+    pss_status rc = validate_batch(h, indices, nnz, offsets, B);
+    if (rc != PSS_OK) return rc;
+    const int64_t nbags = (int64_t)h->dp.T * B;
+    if (nbags > 0 && !out) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int64_t *di = nullptr, *doff = nullptr;
+    if ((rc = device_view(indices, (size_t)nnz, h->st_idx, st, &di)) != PSS_OK) return rc;
+    if ((rc = device_view(offsets, (size_t)(nbags + 1), h->st_off, st, &doff)) != PSS_OK) return rc;
+    const size_t nout = (size_t)nbags * (size_t)h->dp.d;
+    float* dout = out;
+    const bool host_out = nout > 0 && !is_device_ptr(out);
+    if (host_out) {
+        PSS_TRY(ensure(h->st_out, nout * sizeof(float), st));
+        dout = static_cast<float*>(h->st_out.ptr);
+    }
+    if (nbags > 0) {
+        LaunchScope ls(h, PSS_K_FORWARD, st);
+        PSS_TRY(launch_forward(h->dp, layout_for(h, dout), di, nnz, doff, B, h->w, dout, h->err,
+                               h->sm_count, st));
+    }
+    if (host_out)
+        PSS_TRY(cudaMemcpyAsync(out, dout, nout * sizeof(float), cudaMemcpyDeviceToHost, st));
+    h->last_idx = di;
+    h->last_off = doff;
+    h->last_nnz = nnz;
+    h->last_B = B;
+    h->have_batch = true;
+    if (h->sync_check) return check_error_word(h, st, nullptr);
+    return PSS_OK;
+}
+
+static pss_status scatter_into(pss_handle* h, const float* dgrad, float scale, float* target,
+                               bool touch, cudaStream_t st) {
+    const int64_t nbags = (int64_t)h->dp.T * h->last_B;
+    if (nbags == 0) return PSS_OK;
+    // 16-byte vector atomics need both the gradient rows and the target aligned
+    RowLayout lay = layout_for(h, dgrad);
+    if (lay.vw == 4 && !aligned16(target)) lay = choose_layout(h->dp.d, 1, 1);
+    LaunchScope ls(h, PSS_K_SCATTER, st);
+    return cuda_status(launch_scatter(h->dp, lay, h->last_idx, h->last_nnz,
+                                      h->last_off, h->last_B, dgrad, scale, target,
+                                      touch ? &h->touched : nullptr, h->err, h->sm_count, st));
+}
+
+pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, pss_stream stream) {
+    if (!h) return PSS_ERR_INVALID_ARG;
+    if (!h->have_batch) return PSS_ERR_STATE;
+    const int64_t nbags = (int64_t)h->dp.T * h->last_B;
+    if (nbags > 0 && !grad_out) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const float* dg = nullptr;
+    pss_status rc = device_view(grad_out, (size_t)nbags * (size_t)h->dp.d, h->st_grad, st, &dg);
+    if (rc != PSS_OK) return rc;
+    const int64_t pairs = h->last_nnz * (int64_t)h->dp.J;
+    h->last_path = PSS_PATH_ATOMIC;
+    if (h->opt == PSS_SGD) {
+        // SGD is linear in g: scatter -lr * grad_out straight into M.
+        if (lr != 0.f && (rc = scatter_into(h, dg, -lr, h->w, false, st)) != PSS_OK) return rc;
+    } else {
+        if ((rc = ensure_grad(h, st)) != PSS_OK) return rc;
+        const bool touch = use_touched(h, pairs);
+        if (touch && (rc = ensure_touched(h, pairs, st)) != PSS_OK) return rc;
+        if ((rc = scatter_into(h, dg, 1.0f, h->g, touch, st)) != PSS_OK) return rc;
+        {
+            LaunchScope ls(h, PSS_K_UPDATE, st);
+            if (touch)
+                PSS_TRY(launch_update_touched(true, h->w, h->Gacc, h->g, h->touched, h->dp.G,
+                                              h->dp.L, lr, h->eps, h->sm_count, st));
+            else
+                PSS_TRY(launch_adagrad_dense(h->w, h->Gacc, h->g, h->dp.M, lr, h->eps,
+                                             h->sm_count, st));
+        }
+        if (touch) {
+            LaunchScope ls(h, PSS_K_MISC, st);
+            PSS_TRY(launch_touched_clear(h->touched, h->sm_count, st));
+        }
+    }
+    if (h->sync_check) return check_error_word(h, st, nullptr);
+    return PSS_OK;
+}
+
+pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, pss_stream stream) {
+    if (!h || !grad) return PSS_ERR_INVALID_ARG;
+    if (!h->have_batch) return PSS_ERR_STATE;
+    const int64_t nbags = (int64_t)h->dp.T * h->last_B;
+    if (nbags > 0 && !grad_out) return PSS_ERR_INVALID_ARG;
+    if (!is_device_ptr(grad)) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const float* dg = nullptr;
+    pss_status rc = device_view(grad_out, (size_t)nbags * (size_t)h->dp.d, h->st_grad, st, &dg);
+    if (rc != PSS_OK) return rc;
+    PSS_TRY(cudaMemsetAsync(grad, 0, sizeof(float) * (size_t)h->dp.M, st));
+    if ((rc = scatter_into(h, dg, 1.0f, grad, false, st)) != PSS_OK) return rc;
+    if (h->sync_check) return check_error_word(h, st, nullptr);
+    return PSS_OK;
+}
+
+pss_status pss_set_option(pss_handle* h, int32_t key, int64_t value) {
+    if (!h) return PSS_ERR_INVALID_ARG;
+    switch (key) {
+        case PSS_OPT_BACKWARD_PATH:
+            if (value < PSS_PATH_AUTO || value > PSS_PATH_SORTED) return PSS_ERR_INVALID_ARG;
+            h->path = value;
+            return PSS_OK;
+        case PSS_OPT_UPDATE_MODE:
+            if (value < PSS_UPDATE_AUTO || value > PSS_UPDATE_TOUCHED) return PSS_ERR_INVALID_ARG;
+            h->update_mode = value;
+            return PSS_OK;
+        case PSS_OPT_PROFILE:
+            if (value != 0 && value != 1) return PSS_ERR_INVALID_ARG;
+            h->profile = value;
+            return PSS_OK;
+        case PSS_OPT_SYNC_CHECK:
+            if (value != 0 && value != 1) return PSS_ERR_INVALID_ARG;
+            h->sync_check = value;
+            return PSS_OK;
+    }
+    return PSS_ERR_INVALID_ARG;
+}
+
+pss_status pss_get_option(pss_handle* h, int32_t key, int64_t* value) {
+    if (!h || !value) return PSS_ERR_INVALID_ARG;
+    switch (key) {
+        case PSS_OPT_BACKWARD_PATH: *value = h->path; return PSS_OK;
+        case PSS_OPT_UPDATE_MODE: *value = h->update_mode; return PSS_OK;
+        case PSS_OPT_PROFILE: *value = h->profile; return PSS_OK;
+        case PSS_OPT_SYNC_CHECK: *value = h->sync_check; return PSS_OK;
+    }
+    return PSS_ERR_INVALID_ARG;
+}
+
+pss_status pss_get_error(pss_handle* h, int64_t* first_bad_index, pss_stream stream) {
+    if (!h) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    return check_error_word(h, reinterpret_cast<cudaStream_t>(stream), first_bad_index);
+}
+
+pss_status pss_get_info(pss_handle* h, pss_info* info) {
+    if (!h || !info) return PSS_ERR_INVALID_ARG;
+    info->T = h->dp.T;
+    info->d = h->dp.d;
+    info->M = h->dp.M;
+    info->Z = h->dp.Z;
+    info->G = h->dp.G;
+    info->J = h->dp.J;
+    info->L = h->dp.L;
+    info->R = (int64_t)h->dp.R;
+    info->A = h->dp.A;
+    info->B0 = h->dp.B0;
+    info->optimizer = h->opt;
+    info->kernel_launches = h->launches;
+    info->last_path = h->last_path;
+    info->last_collision_rate = h->last_collision;
+    return PSS_OK;
+}
+
+pss_status pss_get_profile(pss_handle* h, int32_t kernel, int64_t* launches, double* total_ms) {
+    if (!h || kernel < 0 || kernel >= PSS_K_COUNT) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    double tot = 0.0;
+    for (auto& e : h->ev[kernel]) {
+        PSS_TRY(cudaEventSynchronize(e.b));
+        float ms = 0.f;
+        PSS_TRY(cudaEventElapsedTime(&ms, e.a, e.b));
+        tot += ms;
+    }
+    if (launches) *launches = (int64_t)h->ev[kernel].size();
+    if (total_ms) *total_ms = tot;
+    return PSS_OK;
+}
+
+pss_status pss_reset_profile(pss_handle* h) {
+    if (!h) return PSS_ERR_INVALID_ARG;
+    DeviceGuard g(h->device);
+    for (int k = 0; k < PSS_K_COUNT; ++k) {
+        for (auto& e : h->ev[k]) {
+            cudaEventSynchronize(e.b);
+            h->ev_free.push_back(e);
+        }
+        h->ev[k].clear();
+    }
+    return PSS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,67 @@
+// Internal declarations shared by the CUDA translation units of libpss.so.
+// Nothing here is part of the public ABI (include/pss.h is).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace pss {
+
+// Hash and shape parameters as the kernels see them.
+//   bucket x = ((A*key + B0) mod P) mod R,  P = 2^61 - 1,  loc = G*x
+//   Rinv = floor((2^64 - 1) / R) drives the exact "mod R" reduction.
+struct DevParams {
+    uint64_t A, B0, R, Rinv;
+    int64_t G, M;
+    int32_t T, d, Z, J, L;
+    const int64_t* cards;   // device, T entries
+};
+
+// Device error word: smallest id position seen out of range, and flag bits.
+struct DevError {
+    unsigned long long first_bad;   // ULLONG_MAX when clear
+    unsigned int flags;             // kErrOffsets
+    unsigned int pad;
+};
+constexpr unsigned int kErrOffsets = 1u;
+
+// Lane layout of one bag row: VW-wide columns, groups of gs lanes per bag.
+struct RowLayout {
+    int vw;        // 4 (float4 columns) or 1
+    int kc;        // columns per lane
+    int log2gs;    // log2(lanes per bag group)
+};
+RowLayout choose_layout(int d, int Z, int64_t G);
+
+// Touched-block bookkeeping for the sparse optimizer pass.
+struct Touched {
+    uint32_t* bitmap;                 // R bits
+    int64_t* list;                    // bucket indices x, capacity cap
+    unsigned long long* count;        // number of entries in list
+    int64_t cap;
+};
+
+// Kernel launchers (return the CUDA launch error).  `grid_cap` bounds the
+// grid of grid-stride kernels; 0 lets the launcher decide.
+cudaError_t launch_locations(const DevParams& p, const int64_t* idx, int64_t nnz,
+                             const int64_t* off, int64_t B, int64_t* locs, DevError* err,
+                             int sm_count, cudaStream_t st);
+cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
+                           int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
+                           DevError* err, int sm_count, cudaStream_t st);
+cudaError_t launch_scatter(const DevParams& p, const RowLayout& lay, const int64_t* idx,
+                           int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
+                           float scale, float* target, const Touched* touched, DevError* err,
+                           int sm_count, cudaStream_t st);
+cudaError_t launch_adagrad_dense(float* w, float* Gacc, float* g, int64_t M, float lr, float eps,
+                                 int sm_count, cudaStream_t st);
+cudaError_t launch_sgd_dense(float* w, float* g, int64_t M, float lr, int sm_count,
+                             cudaStream_t st);
+// Touched-block optimizer pass (one warp per distinct block start), then the
+// pass that clears the bitmap words of the listed starts and resets the count.
+cudaError_t launch_update_touched(bool adagrad, float* w, float* Gacc, float* g,
+                                  const Touched& touched, int64_t G, int32_t L, float lr,
+                                  float eps, int sm_count, cudaStream_t st);
+cudaError_t launch_touched_clear(const Touched& touched, int sm_count, cudaStream_t st);
+
+}  // namespace pss

@@ -1,0 +1,448 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the
+same seeded inputs.
+
+* hash locations: bit-exact;
+* pooled forward: within 1e-6 of sum|terms| (bit-exact on dyadic inputs);
+* gradient (Algorithm 1 dense branch): within 1e-5 of sum|contributions|;
+* updated shared array and Adagrad accumulator: the derived bounds in gpu_util.
+
+Sizes: small cases that span many thread blocks and a ragged tail, then the
+named workloads at full size (tiny, Criteo-Kaggle, Criteo-TB, multi-hot
+contention, the compression sweep), in the default launch configuration that
+bench.py times.
+"""
+import numpy as np
+import pytest
+
+from paper_2207_10731_gb300 import binding, workloads as wl
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+
+def _batch_cuda(w):
+    return gu.cuda(w.indices), gu.cuda(w.offsets)
+
+
+def _abs_pool(o, w_host, w):
+    out, _ = o.forward(np.abs(w_host), w.indices, w.offsets, w.B)
+    return out
+
+
+# --------------------------------------------------------------------------
+# hash (row a2): bit-exact
+LOC_CASES = [
+    dict(name="tiny"),
+    dict(name="kaggle"),
+    dict(name="tb", B=4096),
+    dict(name="multihot", B=512),
+    dict(name="tiny", G=1),                 # paper-literal offsets, scalar path
+    dict(name="tiny", Z=1, G=1),            # HashedNet (Z = 1)
+    dict(name="kaggle", Z=3, G=2, B=300),   # odd chunk, ragged tail
+]
+
+
+@pytest.mark.parametrize("case", LOC_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_locations_bit_exact(case):
+    case = dict(case)
+    w = wl.make_workload(case.pop("name"), grad="none", **case)
+    h, o = gu.make_pair(w)
+    idx, off = _batch_cuda(w)
+    got = gu.host(h.compute_locations(idx, off, w.B))
+    want, bad = o.locations(w.indices, w.offsets, w.B)
+    assert bad == -1
+    np.testing.assert_array_equal(got, want)
+    assert h.get_error() == (binding.PSS_OK, -1)
+    h.close()
+
+
+def test_locations_beyond_32_bits():
+    # M > 2^32 elements: block starts need 64-bit offsets.
+    w = wl.make_workload("tb", B=2048, M=(1 << 33), grad="none")
+    h = binding.PSS(w.cards, dim=w.d, M=w.M, Z=w.Z, G=w.G, seed=0)
+    from oracle import OraclePSS
+    o = OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=0)
+    got = gu.host(h.compute_locations(*_batch_cuda(w), w.B))
+    want, _ = o.locations(w.indices, w.offsets, w.B)
+    np.testing.assert_array_equal(got, want)
+    assert got.max() > (1 << 32)
+    h.close()
+
+
+# --------------------------------------------------------------------------
+# forward (row a3)
+FWD_CASES = [
+    dict(name="tiny"),
+    dict(name="kaggle"),
+    dict(name="tb", B=8192),
+    dict(name="multihot", B=2048),
+    dict(name="multihot", B=777, bag=("uniform", 0, 6)),      # empty bags, ragged tail
+    dict(name="tiny", G=1),
+    dict(name="tiny", Z=1, G=1),
+    dict(name="kaggle", Z=3, G=2, B=300),
+    dict(name="tb", B=1000, d=200, Z=32),                    # two columns per lane
+    dict(name="tb", B=500, d=10, Z=4, G=4),                  # d not a multiple of 4
+]
+
+
+def _wl(case):
+    case = dict(case)
+    name = case.pop("name")
+    over = {k: case.pop(k) for k in ("bag", "d") if k in case}
+    return wl.make_workload(name, **case, **over)
+
+
+@pytest.mark.parametrize("case", FWD_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_forward_parity(case):
+    w = _wl(case)
+    h, o = gu.make_pair(w)
+    out = gu.host(h.forward(*_batch_cuda(w), w.B)).ravel()
+    ref, bad = o.forward(w.w0, w.indices, w.offsets, w.B)
+    assert bad == -1
+    gu.check_forward(out, ref, _abs_pool(o, w.w0, w))
+    h.close()
+
+
+@pytest.mark.parametrize("name,B", [("tiny", 256), ("kaggle", 2048), ("multihot", 1024)])
+def test_forward_dyadic_bit_exact(name, B):
+    w = wl.make_workload(name, B=B, w0="dyadic")
+    h, o = gu.make_pair(w)
+    out = gu.host(h.forward(*_batch_cuda(w), w.B)).ravel()
+    ref, _ = o.forward(w.w0, w.indices, w.offsets, w.B)
+    np.testing.assert_array_equal(out, ref)
+    h.close()
+
+
+# --------------------------------------------------------------------------
+# gradient (row a4): lr = 0 capture through pss_backward_grad
+@pytest.mark.parametrize("case", FWD_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_grad_parity(case):
+    w = _wl(case)
+    h, o = gu.make_pair(w)
+    h.forward(*_batch_cuda(w), w.B)
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    ref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
+    A = o.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g, ref, A)
+    # total mass: sum over bags of |bag| * sum of its upstream gradient row
+    lengths = np.diff(w.offsets).reshape(w.T, w.B)
+    rows = w.grad_out.reshape(w.B, w.T, w.d).astype(np.float64).sum(axis=2)
+    mass = float((lengths.T * rows).sum())
+    assert abs(g.astype(np.float64).sum() - mass) <= 1e-5 * A.sum() + 1e-6
+    h.close()
+
+
+def test_grad_dyadic_and_all_ones_exact():
+    for grad in ("dyadic", "ones"):
+        w = wl.make_workload("kaggle", B=1024, grad=grad, w0="dyadic")
+        h, o = gu.make_pair(w)
+        h.forward(*_batch_cuda(w), w.B)
+        g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+        ref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
+        np.testing.assert_array_equal(g.astype(np.float64), ref)
+        h.close()
+
+
+# --------------------------------------------------------------------------
+# fused backward + optimizer step (rows a4, a5)
+STEP_CASES = [
+    dict(name="tiny"),                                  # SGD lr 0.1
+    dict(name="kaggle"),                                # Adagrad
+    dict(name="tb", B=8192),                            # Adagrad
+    dict(name="multihot", B=2048),                      # SGD, contention
+    dict(name="kaggle", opt="sgd"),
+    dict(name="tiny", opt="adagrad", lr=0.05),
+    dict(name="multihot", B=777, bag=("uniform", 0, 6), opt="adagrad"),
+    dict(name="tiny", G=1, opt="adagrad"),
+    dict(name="tiny", Z=1, G=1),
+]
+
+
+def _run_step(w, h, o, wcur, Gcur, batch):
+    idx, off, go = batch
+    B = (off.shape[0] - 1) // w.T
+    h.forward(gu.cuda(idx), gu.cuda(off), B)
+    h.backward_update(gu.cuda(go), w.lr)
+    wg, Gg = h.get_state()
+    w2, G2, g32 = o.step(wcur, Gcur, idx, off, B, go, w.opt, w.lr, w.eps)
+    A = o.grad(idx, off, B, np.abs(go))
+    return gu.host(wg), (gu.host(Gg) if Gg is not None else None), w2, G2, g32, A
+
+
+@pytest.mark.parametrize("case", STEP_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_step_parity_three_steps(case):
+    case = dict(case)
+    opt = case.pop("opt", None)
+    lr = case.pop("lr", None)
+    w = _wl(case)
+    if opt:
+        w.opt = opt
+    if lr:
+        w.lr = lr
+    h, o = gu.make_pair(w)
+    wcur = w.w0.copy()
+    Gcur = np.zeros(w.M, dtype=np.float32)
+    cfg = wl.CONFIGS[case["name"]]
+    for step in range(3):
+        if step == 0:
+            batch = (w.indices, w.offsets, w.grad_out)
+        else:
+            batch = wl.make_batch(w.cards, w.B, w.d, case.get("bag", cfg["bag"]), cfg["ids"],
+                                  seed=w.seed, batch=step)
+        wg, Gg, wcur_next, Gnext, g32, A = _run_step(w, h, o, wcur, Gcur, batch)
+        if w.opt == "sgd":
+            gu.check_sgd(wg, wcur_next, A, w.lr, what=f"sgd step {step}")
+        else:
+            gu.check_adagrad(wg, Gg, wcur_next, Gnext, g32, A, w.lr, what=f"adagrad step {step}")
+        # continue from the GPU's own state so the steps stay comparable
+        wcur, Gcur = wg.copy(), (Gg.copy() if Gg is not None else Gcur)
+        h.set_state(gu.cuda(wcur), gu.cuda(Gcur) if w.opt == "adagrad" else None)
+    h.close()
+
+
+@pytest.mark.parametrize("opt", ["sgd", "adagrad"])
+def test_step_dyadic_bit_exact(opt):
+    w = wl.make_workload("kaggle", B=1024, grad="dyadic", w0="dyadic")
+    w.lr = 0.125
+    h, o = gu.make_pair(w, opt=opt)
+    h.forward(*_batch_cuda(w), w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    wg, Gg = h.get_state()
+    w2, G2, _ = o.step(w.w0, np.zeros(w.M, np.float32), w.indices, w.offsets, w.B, w.grad_out,
+                       opt, w.lr, w.eps)
+    np.testing.assert_array_equal(gu.host(wg), w2)
+    if opt == "adagrad":
+        np.testing.assert_array_equal(gu.host(Gg), G2)
+    h.close()
+
+
+def test_dense_and_touched_updates_identical():
+    # Same exact gradient (dyadic inputs), two ways of visiting M: same bits.
+    w = wl.make_workload("tb", B=2048, grad="dyadic", w0="dyadic")
+    res = []
+    for mode in (binding.UPDATE_DENSE, binding.UPDATE_TOUCHED):
+        h, _ = gu.make_pair(w, opt="adagrad")
+        h.set_option(binding.OPT_UPDATE_MODE, mode)
+        for _ in range(2):
+            h.forward(*_batch_cuda(w), w.B)
+            h.backward_update(gu.cuda(w.grad_out), 0.01)
+        wg, Gg = h.get_state()
+        res.append((gu.host(wg), gu.host(Gg)))
+        h.close()
+    np.testing.assert_array_equal(res[0][0], res[1][0])
+    np.testing.assert_array_equal(res[0][1], res[1][1])
+
+
+# --------------------------------------------------------------------------
+# full sizes of the named workloads (default launch configuration)
+@pytest.mark.parametrize("name", ["tiny", "kaggle", "tb", "multihot", "microbench"])
+def test_full_size_step(name):
+    w = wl.make_workload(name)
+    h, o = gu.make_pair(w)
+    idx, off = _batch_cuda(w)
+    out = gu.host(h.forward(idx, off, w.B)).ravel()
+    ref, bad = o.forward(w.w0, w.indices, w.offsets, w.B)
+    assert bad == -1
+    gu.check_forward(out, ref, _abs_pool(o, w.w0, w), what=f"{name} forward")
+    del out, ref
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    wg, Gg = h.get_state()
+    w2, G2, g32 = o.step(w.w0, np.zeros(w.M, np.float32), w.indices, w.offsets, w.B, w.grad_out,
+                         w.opt, w.lr, w.eps)
+    A = o.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    if w.opt == "sgd":
+        gu.check_sgd(gu.host(wg), w2, A, w.lr, what=f"{name} sgd")
+    else:
+        gu.check_adagrad(gu.host(wg), gu.host(Gg), w2, G2, g32, A, w.lr, what=f"{name} adagrad")
+    assert h.get_error() == (binding.PSS_OK, -1)
+    h.close()
+
+
+def _sub_batch(w, rows):
+    """Bags of the given batch rows, all tables, as a smaller batch."""
+    rows = np.asarray(rows)
+    idx_parts, lens = [], []
+    for t in range(w.T):
+        for b in rows:
+            s = t * w.B + b
+            seg = w.indices[w.offsets[s]:w.offsets[s + 1]]
+            idx_parts.append(seg)
+            lens.append(seg.shape[0])
+    off = np.zeros(len(lens) + 1, dtype=np.int64)
+    np.cumsum(lens, out=off[1:])
+    return np.concatenate(idx_parts).astype(np.int64), off
+
+
+@pytest.mark.parametrize("logM", [18, 20, 22, 24, 26, 28, 30, 32, 33])
+def test_compression_sweep(logM):
+    """Criteo-TB shape with M from 2^18 to 2^33 fp32 (1 MB .. 32 GB).  Up to
+    2^26 everything is compared; above, sampled rows and sampled elements
+    (touched and untouched) are compared with the oracle evaluated one by one."""
+    t = gu.torch()
+    M = 1 << logM
+    w = wl.make_workload("sweep", M=M)
+    h, o = gu.make_pair(w)
+    idx, off = _batch_cuda(w)
+    out = h.forward(idx, off, w.B)
+    rng = np.random.default_rng(logM)
+    rows = np.sort(rng.choice(w.B, size=64, replace=False))
+    sidx, soff = _sub_batch(w, rows)
+    w0s = w.w0 if w.w0 is not None else None
+    if w0s is not None:
+        ref, _ = o.forward(w0s, sidx, soff, rows.shape[0])
+        absr, _ = o.forward(np.abs(w0s), sidx, soff, rows.shape[0])
+    else:
+        # evaluate the oracle on a compact copy of the touched blocks only
+        locs, _ = o.locations(sidx, soff, rows.shape[0])
+        elems = np.unique((locs[:, None] + np.arange(o.L)[None, :]).ravel())
+        vals = w.w0_at(elems)
+        pos = {int(e): k for k, e in enumerate(elems)}
+        ref = np.zeros(rows.shape[0] * w.T * w.d, np.float64)
+        absr = np.zeros_like(ref)
+        for tt in range(w.T):
+            for bi in range(rows.shape[0]):
+                s = tt * rows.shape[0] + bi
+                for q in range(soff[s], soff[s + 1]):
+                    for j in range(o.J):
+                        base = locs[q * o.J + j]
+                        for z in range(min(w.Z, w.d - j * w.Z)):
+                            v = vals[pos[int(base + z)]]
+                            ref[(bi * w.T + tt) * w.d + j * w.Z + z] += v
+                            absr[(bi * w.T + tt) * w.d + j * w.Z + z] += abs(v)
+    got = gu.host(out[t.from_numpy(rows).cuda()]).ravel()
+    gu.check_forward(got, ref, absr, what=f"sweep 2^{logM} forward")
+    del out
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    if logM <= 26:
+        wg, Gg = h.get_state()
+        w2, G2, g32 = o.step(w.w0, np.zeros(w.M, np.float32), w.indices, w.offsets, w.B,
+                             w.grad_out, w.opt, w.lr, w.eps)
+        A = o.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+        gu.check_adagrad(gu.host(wg), gu.host(Gg), w2, G2, g32, A, w.lr,
+                         what=f"sweep 2^{logM}")
+    else:
+        locs, _ = o.locations(w.indices, w.offsets, w.B)
+        pick = rng.choice(locs.shape[0], size=3000, replace=False)
+        touched = (locs[pick][:, None] + np.arange(o.L)[None, :]).ravel()
+        elems = np.unique(np.concatenate([touched, rng.integers(0, M, 20000)]))
+        g_at = o.grad_at(w.indices, w.offsets, w.B, w.grad_out, elems)
+        A_at = o.grad_at(w.indices, w.offsets, w.B, np.abs(w.grad_out), elems)
+        w_s = w.w0_at(elems).astype(np.float32).copy()
+        G_s = np.zeros(elems.shape[0], np.float32)
+        g32 = g_at.astype(np.float32)
+        o.adagrad(w_s, G_s, g32, w.lr, w.eps)
+        wg, Gg = h.get_state()
+        sel = t.from_numpy(elems).cuda()
+        gu.check_adagrad(gu.host(wg[sel]), gu.host(Gg[sel]), w_s, G_s, g32, A_at, w.lr,
+                         what=f"sweep 2^{logM} sampled")
+        del wg, Gg
+    assert h.get_error() == (binding.PSS_OK, -1)
+    h.close()
+    t.cuda.empty_cache()
+
+
+# --------------------------------------------------------------------------
+# host buffers through the same C-ABI calls (the end-to-end path)
+def test_host_buffers_match_device_buffers():
+    # dyadic inputs: every sum is exact, so both paths must give the same bits
+    t = gu.torch()
+    w = wl.make_workload("kaggle", grad="dyadic", w0="dyadic")
+    w.lr = 0.125
+    h1, _ = gu.make_pair(w, opt="sgd")
+    h2, _ = gu.make_pair(w, opt="sgd")
+    out_d = gu.host(h1.forward(*_batch_cuda(w), w.B))
+    idx_h = t.from_numpy(w.indices).pin_memory()
+    off_h = t.from_numpy(w.offsets).pin_memory()
+    out_h = h2.forward(idx_h, off_h, w.B)
+    t.cuda.synchronize()
+    assert not out_h.is_cuda
+    np.testing.assert_array_equal(out_h.numpy(), out_d)
+    # pageable host memory works too
+    out_p = t.empty(out_h.shape, dtype=t.float32)
+    h2.forward(t.from_numpy(w.indices), t.from_numpy(w.offsets), w.B, out=out_p)
+    t.cuda.synchronize()
+    np.testing.assert_array_equal(out_p.numpy(), out_d)
+    h1.backward_update(gu.cuda(w.grad_out), w.lr)
+    h2.backward_update(t.from_numpy(w.grad_out).pin_memory(), w.lr)
+    np.testing.assert_array_equal(gu.host(h2.get_weights()), gu.host(h1.get_weights()))
+    h1.close()
+    h2.close()
+
+
+# --------------------------------------------------------------------------
+# errors: reported, never a trap
+def test_out_of_range_ids_are_skipped_and_reported():
+    w = wl.make_workload("tiny")
+    idx = w.indices.copy()
+    idx[100] = 5000          # beyond the 1000-id table
+    idx[37] = -3
+    h, o = gu.make_pair(w)
+    out = gu.host(h.forward(gu.cuda(idx), gu.cuda(w.offsets), w.B)).ravel()
+    st, first = h.get_error()
+    assert st == binding.PSS_ERR_INDEX_RANGE and first == 37
+    ref, bad = o.forward(w.w0, idx, w.offsets, w.B)
+    assert bad == 37
+    np.testing.assert_array_equal(out, ref)
+    assert h.get_error() == (binding.PSS_OK, -1)     # cleared by the read
+    h.close()
+
+
+def test_malformed_offsets_reported():
+    w = wl.make_workload("tiny")
+    off = w.offsets.copy()
+    off[10] = off[11] + 5    # decreasing
+    h, _ = gu.make_pair(w)
+    h.forward(gu.cuda(w.indices), gu.cuda(off), w.B)
+    st, first = h.get_error()
+    assert st == binding.PSS_ERR_INDEX_RANGE and first == -2
+    h.close()
+
+
+def test_call_order_and_argument_errors():
+    w = wl.make_workload("tiny")
+    h, _ = gu.make_pair(w)
+    with pytest.raises(binding.PSSError) as e:
+        h.backward_update(gu.cuda(w.grad_out), 0.1)
+    assert e.value.status == binding.PSS_ERR_STATE
+    with pytest.raises(binding.PSSError) as e:
+        h.set_weights(gu.cuda(np.zeros(10, np.float32)))
+    assert e.value.status == binding.PSS_ERR_INVALID_ARG
+    with pytest.raises(binding.PSSError):
+        h.set_option(99, 0)
+    with pytest.raises(binding.PSSError):
+        h.set_option(binding.OPT_BACKWARD_PATH, 7)
+    h.close()
+
+
+def test_empty_batch():
+    w = wl.make_workload("tiny")
+    h, _ = gu.make_pair(w)
+    t = gu.torch()
+    out = h.forward(t.zeros(0, dtype=t.int64, device="cuda"),
+                    t.zeros(1, dtype=t.int64, device="cuda"), 0)
+    assert out.numel() == 0
+    h.backward_update(t.zeros(0, dtype=t.float32, device="cuda"), 0.1)
+    wg = gu.host(h.get_weights())
+    np.testing.assert_array_equal(wg, w.w0)
+    # bags that are all empty: zero rows, no update
+    off = np.zeros(w.T * 4 + 1, np.int64)
+    out = gu.host(h.forward(t.zeros(0, dtype=t.int64, device="cuda"), gu.cuda(off), 4))
+    assert out.shape == (4, w.T, w.d) and not out.any()
+    h.close()
+
+
+def test_profile_and_launch_counts():
+    w = wl.make_workload("kaggle")
+    h, _ = gu.make_pair(w)
+    h.set_option(binding.OPT_PROFILE, 1)
+    idx, off = _batch_cuda(w)
+    go = gu.cuda(w.grad_out)
+    before = h.info()["kernel_launches"]
+    for _ in range(3):
+        h.forward(idx, off, w.B)
+        h.backward_update(go, w.lr)
+    n_f, ms_f = h.profile(binding.K_FORWARD)
+    n_s, ms_s = h.profile(binding.K_SCATTER)
+    assert n_f == 3 and n_s == 3 and ms_f > 0 and ms_s > 0
+    assert h.info()["kernel_launches"] - before == 9     # forward, scatter, update
+    h.close()
