@@ -203,7 +203,7 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    w = wl.make_workload(args.workload, M=args.M)
+    w = wl.make_workload(args.workload, M=args.M, B=args.B)
     import oracle
     o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed)
     total_budget = 90.0
@@ -261,7 +261,7 @@ def run_gpu(args):
         dist.init_process_group("nccl", device_id=dev)
 
     # one replica per rank, each with its own batch (no data-path exchange)
-    w = wl.make_workload(args.workload, seed=0, M=args.M)
+    w = wl.make_workload(args.workload, seed=0, M=args.M, B=args.B)
     batches = [(w.indices, w.offsets, w.grad_out)]
     for k in range(1, args.rotate):
         batches.append(wl.make_batch(w.cards, w.B, w.d, wl.CONFIGS[args.workload]["bag"],
@@ -277,6 +277,7 @@ def run_gpu(args):
         base = torch.from_numpy(w.w0_base).to(dev)
         h.set_weights(base.repeat(-(-w.M // base.numel()))[: w.M].contiguous())
         del base
+    h.set_option(binding.OPT_ACCUM, binding.ACCUM_F32 if args.accum == "f32" else binding.ACCUM_F64)
     out = torch.empty((w.B, w.T, w.d), dtype=torch.float32, device=dev)
     nnz_per_step = [int(b[0].shape[0]) for b in batches]
     stream = torch.cuda.current_stream()
@@ -387,6 +388,7 @@ def run_gpu(args):
             "config": {"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B * world,
                        "seq_len": 1,
                        "parallelism": "independent replicas" if world > 1 else "single GPU",
+                       "grad_accumulator": args.accum,
                        "l2": (f"inputs larger than L2: {args.rotate}-batch rotation, "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB output and "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB upstream gradient per step")},
@@ -425,6 +427,9 @@ def main(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle timing")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--accum", choices=["f64", "f32"], default="f64",
+                    help="gradient accumulator precision of the atomic path")
+    ap.add_argument("--B", type=int, default=None, help="override the batch size (profiling)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")

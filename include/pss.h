@@ -88,8 +88,18 @@ typedef enum {
     PSS_OPT_PROFILE = 3,
     /* 1: forward/backward synchronise the stream and return
      * PSS_ERR_INDEX_RANGE at once when the device error word is set. */
-    PSS_OPT_SYNC_CHECK = 4
+    PSS_OPT_SYNC_CHECK = 4,
+    /* Precision of the gradient accumulator of the atomic path.
+     * PSS_ACCUM_F64 (default): every contribution is added in fp64 and the sum
+     * is rounded to fp32 once, so the error does not grow with the number of
+     * contributions (8 bytes of scratch per element of M).
+     * PSS_ACCUM_F32: 16-byte fp32 vector reductions (4 bytes per element, and
+     * SGD is scattered straight into M); the error of a recursive fp32 sum,
+     * up to (n-1) * 2^-24 * sum|contributions| for an element with n of them. */
+    PSS_OPT_ACCUM = 5
 } pss_option;
+
+enum { PSS_ACCUM_F64 = 0, PSS_ACCUM_F32 = 1 };
 
 enum { PSS_PATH_AUTO = 0, PSS_PATH_ATOMIC = 1, PSS_PATH_SORTED = 2 };
 enum { PSS_UPDATE_AUTO = 0, PSS_UPDATE_DENSE = 1, PSS_UPDATE_TOUCHED = 2 };

@@ -22,7 +22,8 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libpss.so")
 PSS_OK, PSS_ERR_INVALID_ARG, PSS_ERR_OOM, PSS_ERR_CUDA, PSS_ERR_STATE, PSS_ERR_INDEX_RANGE, \
     PSS_ERR_TIMEOUT, PSS_ERR_UNSUPPORTED = range(8)
 PSS_SGD, PSS_ADAGRAD = 0, 1
-OPT_BACKWARD_PATH, OPT_UPDATE_MODE, OPT_PROFILE, OPT_SYNC_CHECK = 1, 2, 3, 4
+OPT_BACKWARD_PATH, OPT_UPDATE_MODE, OPT_PROFILE, OPT_SYNC_CHECK, OPT_ACCUM = 1, 2, 3, 4, 5
+ACCUM_F64, ACCUM_F32 = 0, 1
 PATH_AUTO, PATH_ATOMIC, PATH_SORTED = 0, 1, 2
 UPDATE_AUTO, UPDATE_DENSE, UPDATE_TOUCHED = 0, 1, 2
 K_LOCATIONS, K_FORWARD, K_SCATTER, K_UPDATE, K_SORT, K_REDUCE, K_MISC = range(7)

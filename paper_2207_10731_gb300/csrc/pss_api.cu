@@ -47,7 +47,8 @@ struct pss_handle {
 
     float* w = nullptr;          // shared array M (library-owned)
     float* Gacc = nullptr;       // Adagrad accumulator
-    float* g = nullptr;          // dense gradient scratch, zero between calls
+    float* g = nullptr;          // fp32 gradient accumulator, zero between calls
+    double* g64 = nullptr;       // fp64 gradient accumulator, zero between calls
     int64_t* cards_dev = nullptr;
     DevError* err = nullptr;
 
@@ -62,6 +63,7 @@ struct pss_handle {
     int64_t update_mode = PSS_UPDATE_AUTO;
     int64_t profile = 0;
     int64_t sync_check = 0;
+    int64_t accum = PSS_ACCUM_F64;
     int64_t last_path = PSS_PATH_ATOMIC;
     double last_collision = -1.0;
 
@@ -176,9 +178,15 @@ pss_status check_error_word(pss_handle* h, cudaStream_t st, int64_t* first_bad) 
 }
 
 pss_status ensure_grad(pss_handle* h, cudaStream_t st) {
-    if (h->g) return PSS_OK;
-    PSS_TRY(cudaMalloc(&h->g, sizeof(float) * (size_t)h->dp.M));
-    PSS_TRY(cudaMemsetAsync(h->g, 0, sizeof(float) * (size_t)h->dp.M, st));
+    if (h->accum == PSS_ACCUM_F32) {
+        if (h->g) return PSS_OK;
+        PSS_TRY(cudaMalloc(&h->g, sizeof(float) * (size_t)h->dp.M));
+        PSS_TRY(cudaMemsetAsync(h->g, 0, sizeof(float) * (size_t)h->dp.M, st));
+        return PSS_OK;
+    }
+    if (h->g64) return PSS_OK;
+    PSS_TRY(cudaMalloc(&h->g64, sizeof(double) * (size_t)h->dp.M));
+    PSS_TRY(cudaMemsetAsync(h->g64, 0, sizeof(double) * (size_t)h->dp.M, st));
     return PSS_OK;
 }
 
@@ -334,6 +342,7 @@ pss_status pss_destroy(pss_handle* h) {
     cudaFree(h->w);
     cudaFree(h->Gacc);
     cudaFree(h->g);
+    cudaFree(h->g64);
     cudaFree(h->cards_dev);
     cudaFree(h->err);
     cudaFree(h->touched.bitmap);
@@ -457,6 +466,15 @@ pss_status pss_forward(pss_handle* h, const int64_t* indices, int64_t nnz, const
     return PSS_OK;
 }
 
+static pss_status scatter_into64(pss_handle* h, const float* dgrad, bool touch, cudaStream_t st) {
+    const int64_t nbags = (int64_t)h->dp.T * h->last_B;
+    if (nbags == 0) return PSS_OK;
+    LaunchScope ls(h, PSS_K_SCATTER, st);
+    return cuda_status(launch_scatter64(h->dp, layout_for(h, dgrad), h->last_idx, h->last_nnz,
+                                        h->last_off, h->last_B, dgrad, h->g64,
+                                        touch ? &h->touched : nullptr, h->err, h->sm_count, st));
+}
+
 static pss_status scatter_into(pss_handle* h, const float* dgrad, float scale, float* target,
                                bool touch, cudaStream_t st) {
     const int64_t nbags = (int64_t)h->dp.T * h->last_B;
@@ -481,23 +499,37 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
     pss_status rc = device_view(grad_out, (size_t)nbags * (size_t)h->dp.d, h->st_grad, st, &dg);
     if (rc != PSS_OK) return rc;
     const int64_t pairs = h->last_nnz * (int64_t)h->dp.J;
+    const bool ada = h->opt == PSS_ADAGRAD;
     h->last_path = PSS_PATH_ATOMIC;
-    if (h->opt == PSS_SGD) {
+    if (h->accum == PSS_ACCUM_F32 && !ada) {
         // SGD is linear in g: scatter -lr * grad_out straight into M.
         if (lr != 0.f && (rc = scatter_into(h, dg, -lr, h->w, false, st)) != PSS_OK) return rc;
     } else {
         if ((rc = ensure_grad(h, st)) != PSS_OK) return rc;
         const bool touch = use_touched(h, pairs);
         if (touch && (rc = ensure_touched(h, pairs, st)) != PSS_OK) return rc;
-        if ((rc = scatter_into(h, dg, 1.0f, h->g, touch, st)) != PSS_OK) return rc;
+        if (h->accum == PSS_ACCUM_F32)
+            rc = scatter_into(h, dg, 1.0f, h->g, touch, st);
+        else
+            rc = scatter_into64(h, dg, touch, st);
+        if (rc != PSS_OK) return rc;
         {
             LaunchScope ls(h, PSS_K_UPDATE, st);
-            if (touch)
-                PSS_TRY(launch_update_touched(true, h->w, h->Gacc, h->g, h->touched, h->dp.G,
-                                              h->dp.L, lr, h->eps, h->sm_count, st));
-            else
-                PSS_TRY(launch_adagrad_dense(h->w, h->Gacc, h->g, h->dp.M, lr, h->eps,
-                                             h->sm_count, st));
+            if (h->accum == PSS_ACCUM_F32) {
+                if (touch)
+                    PSS_TRY(launch_update_touched(ada, h->w, h->Gacc, h->g, h->touched, h->dp.G,
+                                                  h->dp.L, lr, h->eps, h->sm_count, st));
+                else
+                    PSS_TRY(launch_update_dense(ada, h->w, h->Gacc, h->g, h->dp.M, lr, h->eps,
+                                                h->sm_count, st));
+            } else {
+                if (touch)
+                    PSS_TRY(launch_update_touched64(ada, h->w, h->Gacc, h->g64, h->touched,
+                                                    h->dp.G, h->dp.L, lr, h->eps, h->sm_count, st));
+                else
+                    PSS_TRY(launch_update_dense64(ada, h->w, h->Gacc, h->g64, h->dp.M, lr, h->eps,
+                                                  h->sm_count, st));
+            }
         }
         if (touch) {
             LaunchScope ls(h, PSS_K_MISC, st);
@@ -519,8 +551,15 @@ pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, 
     const float* dg = nullptr;
     pss_status rc = device_view(grad_out, (size_t)nbags * (size_t)h->dp.d, h->st_grad, st, &dg);
     if (rc != PSS_OK) return rc;
-    PSS_TRY(cudaMemsetAsync(grad, 0, sizeof(float) * (size_t)h->dp.M, st));
-    if ((rc = scatter_into(h, dg, 1.0f, grad, false, st)) != PSS_OK) return rc;
+    if (h->accum == PSS_ACCUM_F32) {
+        PSS_TRY(cudaMemsetAsync(grad, 0, sizeof(float) * (size_t)h->dp.M, st));
+        if ((rc = scatter_into(h, dg, 1.0f, grad, false, st)) != PSS_OK) return rc;
+    } else {
+        if ((rc = ensure_grad(h, st)) != PSS_OK) return rc;
+        if ((rc = scatter_into64(h, dg, false, st)) != PSS_OK) return rc;
+        LaunchScope ls(h, PSS_K_MISC, st);
+        PSS_TRY(launch_grad_export(h->g64, grad, h->dp.M, h->sm_count, st));
+    }
     if (h->sync_check) return check_error_word(h, st, nullptr);
     return PSS_OK;
 }
@@ -544,6 +583,10 @@ pss_status pss_set_option(pss_handle* h, int32_t key, int64_t value) {
             if (value != 0 && value != 1) return PSS_ERR_INVALID_ARG;
             h->sync_check = value;
             return PSS_OK;
+        case PSS_OPT_ACCUM:
+            if (value != PSS_ACCUM_F64 && value != PSS_ACCUM_F32) return PSS_ERR_INVALID_ARG;
+            h->accum = value;
+            return PSS_OK;
     }
     return PSS_ERR_INVALID_ARG;
 }
@@ -555,6 +598,7 @@ pss_status pss_get_option(pss_handle* h, int32_t key, int64_t* value) {
         case PSS_OPT_UPDATE_MODE: *value = h->update_mode; return PSS_OK;
         case PSS_OPT_PROFILE: *value = h->profile; return PSS_OK;
         case PSS_OPT_SYNC_CHECK: *value = h->sync_check; return PSS_OK;
+        case PSS_OPT_ACCUM: *value = h->accum; return PSS_OK;
     }
     return PSS_ERR_INVALID_ARG;
 }

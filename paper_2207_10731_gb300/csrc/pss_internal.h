@@ -49,19 +49,31 @@ cudaError_t launch_locations(const DevParams& p, const int64_t* idx, int64_t nnz
 cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
                            DevError* err, int sm_count, cudaStream_t st);
+// Backward scatter into an fp32 target (scale applied to grad_out) or into an
+// fp64 accumulator (scale 1).
 cudaError_t launch_scatter(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
                            float scale, float* target, const Touched* touched, DevError* err,
                            int sm_count, cudaStream_t st);
-cudaError_t launch_adagrad_dense(float* w, float* Gacc, float* g, int64_t M, float lr, float eps,
-                                 int sm_count, cudaStream_t st);
-cudaError_t launch_sgd_dense(float* w, float* g, int64_t M, float lr, int sm_count,
+cudaError_t launch_scatter64(const DevParams& p, const RowLayout& lay, const int64_t* idx,
+                             int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
+                             double* target, const Touched* touched, DevError* err, int sm_count,
                              cudaStream_t st);
-// Touched-block optimizer pass (one warp per distinct block start), then the
-// pass that clears the bitmap words of the listed starts and resets the count.
+// Optimizer passes: dense over M, or over the touched blocks (one warp per
+// distinct block start); g is returned to zero.
+cudaError_t launch_update_dense(bool adagrad, float* w, float* Gacc, float* g, int64_t M,
+                                float lr, float eps, int sm_count, cudaStream_t st);
+cudaError_t launch_update_dense64(bool adagrad, float* w, float* Gacc, double* g, int64_t M,
+                                  float lr, float eps, int sm_count, cudaStream_t st);
 cudaError_t launch_update_touched(bool adagrad, float* w, float* Gacc, float* g,
                                   const Touched& touched, int64_t G, int32_t L, float lr,
                                   float eps, int sm_count, cudaStream_t st);
+cudaError_t launch_update_touched64(bool adagrad, float* w, float* Gacc, double* g,
+                                    const Touched& touched, int64_t G, int32_t L, float lr,
+                                    float eps, int sm_count, cudaStream_t st);
+// out[e] = fp32(g[e]); g[e] = 0 for all e < M.
+cudaError_t launch_grad_export(double* g, float* out, int64_t M, int sm_count, cudaStream_t st);
+// Clears the bitmap words of the listed starts and resets the list count.
 cudaError_t launch_touched_clear(const Touched& touched, int sm_count, cudaStream_t st);
 
 }  // namespace pss

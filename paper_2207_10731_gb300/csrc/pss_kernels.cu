@@ -110,6 +110,31 @@ __device__ __forceinline__ void split_slot(int64_t s, int64_t B, uint64_t Binv, 
     b = (int64_t)r;
 }
 
+// Reduction of one VW-wide column into an fp32 or fp64 accumulator.
+template <int VW, typename AT>
+struct Acc;
+template <int VW>
+struct Acc<VW, float> {
+    static __device__ __forceinline__ void red(float* p, typename Vec<VW>::T v) { Vec<VW>::red(p, v); }
+};
+template <>
+struct Acc<4, double> {
+    static __device__ __forceinline__ void red(double* p, float4 v) {
+        red_add_f64(p + 0, (double)v.x);
+        red_add_f64(p + 1, (double)v.y);
+        red_add_f64(p + 2, (double)v.z);
+        red_add_f64(p + 3, (double)v.w);
+    }
+};
+template <>
+struct Acc<1, double> {
+    static __device__ __forceinline__ void red(double* p, float v) { red_add_f64(p, (double)v); }
+};
+
+// Accumulator element -> fp32 gradient (rounded once, to nearest).
+__device__ __forceinline__ float to_f32(float v) { return v; }
+__device__ __forceinline__ float to_f32(double v) { return __double2float_rn(v); }
+
 __device__ __forceinline__ bool bag_range(const int64_t* __restrict__ off, int64_t s, int64_t nnz,
                                           int64_t& q0, int64_t& q1) {
     q0 = __ldg(off + s);
@@ -218,14 +243,17 @@ __device__ __forceinline__ void mark_touched(const Touched& tc, uint64_t x) {
 
 // ---------------------------------------------------------------------------
 // Backward scatter (dense branch of Algorithm 1): for every id of every bag,
-// add scale * grad_out row chunk j into target[loc(t,i,j) + z].  With
-// target = M and scale = -lr this is the whole SGD step.  TOUCH also records
-// every distinct block start in the touched bitmap/list.
-template <int VW, int KC, bool TOUCH>
+// add scale * grad_out row chunk j into target[loc(t,i,j) + z].  AT = double
+// accumulates in fp64 (one scalar reduction per element: the result is the
+// exact sum up to n*2^-53 relative, rounded once later); AT = float uses 16-byte
+// fp32 vector reductions (recursive fp32 summation in atomic order).  With an
+// fp32 target = M and scale = -lr this is the whole SGD step.  TOUCH also
+// records every distinct block start in the touched bitmap/list.
+template <int VW, int KC, bool TOUCH, typename AT>
 __global__ void __launch_bounds__(kThreads)
 k_scatter(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
           const int64_t* __restrict__ off, int64_t B, uint64_t Binv, const float* __restrict__ gout,
-          float scale, float* target, Touched tc, DevError* err, int log2gs) {
+          float scale, AT* target, Touched tc, DevError* err, int log2gs) {
     using V = Vec<VW>;
     const int lane = threadIdx.x & 31;
     const int gs = 1 << log2gs;
@@ -259,7 +287,7 @@ k_scatter(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
             for (int k = 0; k < KC; ++k) {
                 if (!col.v[k]) continue;
                 const uint64_t x = hash_bucket(p, kb + col.j[k]);
-                V::red(target + G * x + col.z[k], gv[k]);
+                Acc<VW, AT>::red(target + G * x + col.z[k], gv[k]);
                 if (TOUCH && col.z[k] == 0) mark_touched(tc, x);
             }
         }
@@ -281,41 +309,78 @@ __device__ __forceinline__ void adagrad_elem(float& w, float& Ga, float g, float
     Ga = Gn;
 }
 
-template <bool ADA>
+template <typename GT>
+__device__ __forceinline__ bool load4_nonzero(GT* g, int64_t i, float (&gv)[4]);
+template <>
+__device__ __forceinline__ bool load4_nonzero<float>(float* g, int64_t i, float (&gv)[4]) {
+    const float4 v = reinterpret_cast<const float4*>(g)[i];
+    gv[0] = v.x; gv[1] = v.y; gv[2] = v.z; gv[3] = v.w;
+    return v.x != 0.f || v.y != 0.f || v.z != 0.f || v.w != 0.f;
+}
+template <>
+__device__ __forceinline__ bool load4_nonzero<double>(double* g, int64_t i, float (&gv)[4]) {
+    const double2 a = reinterpret_cast<const double2*>(g)[2 * i];
+    const double2 b = reinterpret_cast<const double2*>(g)[2 * i + 1];
+    gv[0] = to_f32(a.x); gv[1] = to_f32(a.y); gv[2] = to_f32(b.x); gv[3] = to_f32(b.y);
+    return a.x != 0.0 || a.y != 0.0 || b.x != 0.0 || b.y != 0.0;
+}
+__device__ __forceinline__ void zero4(float* g, int64_t i) {
+    reinterpret_cast<float4*>(g)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+}
+__device__ __forceinline__ void zero4(double* g, int64_t i) {
+    reinterpret_cast<double2*>(g)[2 * i] = make_double2(0.0, 0.0);
+    reinterpret_cast<double2*>(g)[2 * i + 1] = make_double2(0.0, 0.0);
+}
+
+// Dense pass over M: apply the step where the (rounded) gradient is non-zero
+// and return the accumulator to zero.
+template <bool ADA, typename GT>
 __global__ void __launch_bounds__(kThreads)
-k_update_dense(float* __restrict__ w, float* __restrict__ Ga, float* __restrict__ g, int64_t M,
+k_update_dense(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g, int64_t M,
                float lr, float eps) {
     const int64_t n4 = M >> 2;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     float4* w4 = reinterpret_cast<float4*>(w);
     float4* G4 = reinterpret_cast<float4*>(Ga);
-    float4* g4 = reinterpret_cast<float4*>(g);
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
-        const float4 gv = g4[i];
-        if (gv.x == 0.f && gv.y == 0.f && gv.z == 0.f && gv.w == 0.f) continue;
+        float gv[4];
+        if (!load4_nonzero(g, i, gv)) continue;
         float4 wv = w4[i];
+        float* wp = reinterpret_cast<float*>(&wv);
         if (ADA) {
             float4 Gv = G4[i];
-            if (gv.x != 0.f) adagrad_elem(wv.x, Gv.x, gv.x, lr, eps);
-            if (gv.y != 0.f) adagrad_elem(wv.y, Gv.y, gv.y, lr, eps);
-            if (gv.z != 0.f) adagrad_elem(wv.z, Gv.z, gv.z, lr, eps);
-            if (gv.w != 0.f) adagrad_elem(wv.w, Gv.w, gv.w, lr, eps);
+            float* Gp = reinterpret_cast<float*>(&Gv);
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (gv[c] != 0.f) adagrad_elem(wp[c], Gp[c], gv[c], lr, eps);
             G4[i] = Gv;
         } else {
-            sgd_elem(wv.x, gv.x, lr);
-            sgd_elem(wv.y, gv.y, lr);
-            sgd_elem(wv.z, gv.z, lr);
-            sgd_elem(wv.w, gv.w, lr);
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (gv[c] != 0.f) sgd_elem(wp[c], gv[c], lr);
         }
         w4[i] = wv;
-        g4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        zero4(g, i);
     }
     for (int64_t e = n4 * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < M; e += stride) {
-        const float gv = g[e];
-        if (gv == 0.f) continue;
-        if (ADA) adagrad_elem(w[e], Ga[e], gv, lr, eps);
-        else sgd_elem(w[e], gv, lr);
-        g[e] = 0.f;
+        if (g[e] == (GT)0) continue;
+        const float gv = to_f32(g[e]);
+        if (gv != 0.f) {
+            if (ADA) adagrad_elem(w[e], Ga[e], gv, lr, eps);
+            else sgd_elem(w[e], gv, lr);
+        }
+        g[e] = (GT)0;
+    }
+}
+
+// Gradient export: out[e] = fp32(g[e]) and g[e] = 0, over all of M.
+__global__ void __launch_bounds__(kThreads)
+k_grad_export(double* __restrict__ g, float* __restrict__ out, int64_t M) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < M; e += stride) {
+        const double v = g[e];
+        out[e] = to_f32(v);
+        if (v != 0.0) g[e] = 0.0;
     }
 }
 
@@ -323,9 +388,9 @@ k_update_dense(float* __restrict__ w, float* __restrict__ Ga, float* __restrict_
 // list).  Element e = x*G + z belongs to the LAST marked start at or below it
 // (no marked bucket in (x, x + z/G]), so every element is updated exactly
 // once and without atomics even though blocks overlap when G < L.
-template <bool ADA>
+template <bool ADA, typename GT>
 __global__ void __launch_bounds__(kThreads)
-k_update_touched(float* __restrict__ w, float* __restrict__ Ga, float* __restrict__ g,
+k_update_touched(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g,
                  Touched tc, int64_t G, int L, float lr, float eps) {
     const int lane = threadIdx.x & 31;
     unsigned long long n = *tc.count;
@@ -348,11 +413,14 @@ k_update_touched(float* __restrict__ w, float* __restrict__ Ga, float* __restric
             }
             if (!owner) continue;
             const int64_t e = (int64_t)x * G + z;
-            const float gv = g[e];
-            if (gv == 0.f) continue;
-            if (ADA) adagrad_elem(w[e], Ga[e], gv, lr, eps);
-            else sgd_elem(w[e], gv, lr);
-            g[e] = 0.f;
+            const GT raw = g[e];
+            if (raw == (GT)0) continue;
+            const float gv = to_f32(raw);
+            if (gv != 0.f) {
+                if (ADA) adagrad_elem(w[e], Ga[e], gv, lr, eps);
+                else sgd_elem(w[e], gv, lr);
+            }
+            g[e] = (GT)0;
         }
     }
 }
@@ -377,31 +445,76 @@ cudaError_t forward_inst(const DevParams& p, const RowLayout& lay, const int64_t
     return cudaGetLastError();
 }
 
-template <int VW, int KC, bool TOUCH>
+template <int VW, int KC, bool TOUCH, typename AT>
 cudaError_t scatter_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                          const int64_t* off, int64_t B, const float* gout, float scale,
-                         float* target, const Touched& tc, DevError* err, int sm_count,
+                         AT* target, const Touched& tc, DevError* err, int sm_count,
                          cudaStream_t st) {
     const int64_t nbags = (int64_t)p.T * B;
     const int64_t per_block = (int64_t)kWarps * (32 >> lay.log2gs);
-    const int grid = grid_for(k_scatter<VW, KC, TOUCH>, sm_count,
+    const int grid = grid_for(k_scatter<VW, KC, TOUCH, AT>, sm_count,
                               (nbags + per_block - 1) / per_block);
-    k_scatter<VW, KC, TOUCH><<<grid, kThreads, 0, st>>>(p, idx, nnz, off, B, UINT64_MAX / (uint64_t)B,
-                                                        gout, scale, target, tc, err, lay.log2gs);
+    k_scatter<VW, KC, TOUCH, AT><<<grid, kThreads, 0, st>>>(p, idx, nnz, off, B,
+                                                            UINT64_MAX / (uint64_t)B, gout, scale,
+                                                            target, tc, err, lay.log2gs);
     return cudaGetLastError();
 }
 
-template <int VW, int KC>
+template <int VW, int KC, typename AT>
 cudaError_t scatter_touch(bool touch, const DevParams& p, const RowLayout& lay,
                           const int64_t* idx, int64_t nnz, const int64_t* off, int64_t B,
-                          const float* gout, float scale, float* target, const Touched* tc,
+                          const float* gout, float scale, AT* target, const Touched* tc,
                           DevError* err, int sm_count, cudaStream_t st) {
     Touched none{};
     if (touch)
-        return scatter_inst<VW, KC, true>(p, lay, idx, nnz, off, B, gout, scale, target, *tc, err,
-                                          sm_count, st);
-    return scatter_inst<VW, KC, false>(p, lay, idx, nnz, off, B, gout, scale, target, none, err,
-                                       sm_count, st);
+        return scatter_inst<VW, KC, true, AT>(p, lay, idx, nnz, off, B, gout, scale, target, *tc,
+                                              err, sm_count, st);
+    return scatter_inst<VW, KC, false, AT>(p, lay, idx, nnz, off, B, gout, scale, target, none,
+                                           err, sm_count, st);
+}
+
+template <typename AT>
+cudaError_t scatter_dispatch(const DevParams& p, const RowLayout& lay, const int64_t* idx,
+                             int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
+                             float scale, AT* target, const Touched* touched, DevError* err,
+                             int sm_count, cudaStream_t st) {
+    const bool tch = touched != nullptr;
+#define PSS_SC(VW, KC) \
+    return scatter_touch<VW, KC, AT>(tch, p, lay, idx, nnz, off, B, grad_out, scale, target, \
+                                     touched, err, sm_count, st)
+    if (lay.vw == 4) {
+        switch (lay.kc) {
+            case 1: PSS_SC(4, 1);
+            case 2: PSS_SC(4, 2);
+            case 4: PSS_SC(4, 4);
+        }
+    } else {
+        switch (lay.kc) {
+            case 1: PSS_SC(1, 1);
+            case 2: PSS_SC(1, 2);
+            case 4: PSS_SC(1, 4);
+            case 8: PSS_SC(1, 8);
+            case 16: PSS_SC(1, 16);
+        }
+    }
+#undef PSS_SC
+    return cudaErrorInvalidValue;
+}
+
+template <bool ADA, typename GT>
+cudaError_t update_dense_inst(float* w, float* Ga, GT* g, int64_t M, float lr, float eps,
+                              int sm_count, cudaStream_t st) {
+    const int grid = grid_for(k_update_dense<ADA, GT>, sm_count, ((M >> 2) + kThreads) / kThreads);
+    k_update_dense<ADA, GT><<<grid, kThreads, 0, st>>>(w, Ga, g, M, lr, eps);
+    return cudaGetLastError();
+}
+
+template <bool ADA, typename GT>
+cudaError_t update_touched_inst(float* w, float* Ga, GT* g, const Touched& tc, int64_t G,
+                                int32_t L, float lr, float eps, int sm_count, cudaStream_t st) {
+    const int grid = grid_for(k_update_touched<ADA, GT>, sm_count, (tc.cap + kWarps - 1) / kWarps);
+    k_update_touched<ADA, GT><<<grid, kThreads, 0, st>>>(w, Ga, g, tc, G, L, lr, eps);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -454,53 +567,47 @@ cudaError_t launch_scatter(const DevParams& p, const RowLayout& lay, const int64
                            int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
                            float scale, float* target, const Touched* touched, DevError* err,
                            int sm_count, cudaStream_t st) {
-    const bool tch = touched != nullptr;
-#define PSS_SC(VW, KC) \
-    return scatter_touch<VW, KC>(tch, p, lay, idx, nnz, off, B, grad_out, scale, target, touched, \
-                                 err, sm_count, st)
-    if (lay.vw == 4) {
-        switch (lay.kc) {
-            case 1: PSS_SC(4, 1);
-            case 2: PSS_SC(4, 2);
-            case 4: PSS_SC(4, 4);
-        }
-    } else {
-        switch (lay.kc) {
-            case 1: PSS_SC(1, 1);
-            case 2: PSS_SC(1, 2);
-            case 4: PSS_SC(1, 4);
-            case 8: PSS_SC(1, 8);
-            case 16: PSS_SC(1, 16);
-        }
-    }
-#undef PSS_SC
-    return cudaErrorInvalidValue;
+    return scatter_dispatch<float>(p, lay, idx, nnz, off, B, grad_out, scale, target, touched, err,
+                                   sm_count, st);
 }
 
-cudaError_t launch_adagrad_dense(float* w, float* Ga, float* g, int64_t M, float lr, float eps,
-                                 int sm_count, cudaStream_t st) {
-    const int grid = grid_for(k_update_dense<true>, sm_count, ((M >> 2) + kThreads) / kThreads);
-    k_update_dense<true><<<grid, kThreads, 0, st>>>(w, Ga, g, M, lr, eps);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_sgd_dense(float* w, float* g, int64_t M, float lr, int sm_count,
+cudaError_t launch_scatter64(const DevParams& p, const RowLayout& lay, const int64_t* idx,
+                             int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
+                             double* target, const Touched* touched, DevError* err, int sm_count,
                              cudaStream_t st) {
-    const int grid = grid_for(k_update_dense<false>, sm_count, ((M >> 2) + kThreads) / kThreads);
-    k_update_dense<false><<<grid, kThreads, 0, st>>>(w, nullptr, g, M, lr, 0.f);
-    return cudaGetLastError();
+    return scatter_dispatch<double>(p, lay, idx, nnz, off, B, grad_out, 1.0f, target, touched,
+                                    err, sm_count, st);
+}
+
+cudaError_t launch_update_dense(bool adagrad, float* w, float* Ga, float* g, int64_t M, float lr,
+                                float eps, int sm_count, cudaStream_t st) {
+    return adagrad ? update_dense_inst<true, float>(w, Ga, g, M, lr, eps, sm_count, st)
+                   : update_dense_inst<false, float>(w, Ga, g, M, lr, eps, sm_count, st);
+}
+
+cudaError_t launch_update_dense64(bool adagrad, float* w, float* Ga, double* g, int64_t M,
+                                  float lr, float eps, int sm_count, cudaStream_t st) {
+    return adagrad ? update_dense_inst<true, double>(w, Ga, g, M, lr, eps, sm_count, st)
+                   : update_dense_inst<false, double>(w, Ga, g, M, lr, eps, sm_count, st);
 }
 
 cudaError_t launch_update_touched(bool adagrad, float* w, float* Ga, float* g, const Touched& tc,
                                   int64_t G, int32_t L, float lr, float eps, int sm_count,
                                   cudaStream_t st) {
-    if (adagrad) {
-        const int grid = grid_for(k_update_touched<true>, sm_count, (tc.cap + kWarps - 1) / kWarps);
-        k_update_touched<true><<<grid, kThreads, 0, st>>>(w, Ga, g, tc, G, L, lr, eps);
-    } else {
-        const int grid = grid_for(k_update_touched<false>, sm_count, (tc.cap + kWarps - 1) / kWarps);
-        k_update_touched<false><<<grid, kThreads, 0, st>>>(w, nullptr, g, tc, G, L, lr, 0.f);
-    }
+    return adagrad ? update_touched_inst<true, float>(w, Ga, g, tc, G, L, lr, eps, sm_count, st)
+                   : update_touched_inst<false, float>(w, Ga, g, tc, G, L, lr, eps, sm_count, st);
+}
+
+cudaError_t launch_update_touched64(bool adagrad, float* w, float* Ga, double* g,
+                                    const Touched& tc, int64_t G, int32_t L, float lr, float eps,
+                                    int sm_count, cudaStream_t st) {
+    return adagrad ? update_touched_inst<true, double>(w, Ga, g, tc, G, L, lr, eps, sm_count, st)
+                   : update_touched_inst<false, double>(w, Ga, g, tc, G, L, lr, eps, sm_count, st);
+}
+
+cudaError_t launch_grad_export(double* g, float* out, int64_t M, int sm_count, cudaStream_t st) {
+    const int grid = grid_for(k_grad_export, sm_count, (M + kThreads - 1) / kThreads);
+    k_grad_export<<<grid, kThreads, 0, st>>>(g, out, M);
     return cudaGetLastError();
 }
 

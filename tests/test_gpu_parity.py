@@ -233,6 +233,31 @@ def test_dense_and_touched_updates_identical():
     np.testing.assert_array_equal(res[0][1], res[1][1])
 
 
+@pytest.mark.parametrize("name,B", [("microbench", 10240), ("multihot", 4096), ("tb", 8192)])
+def test_fp32_accumulation_within_recursive_sum_bound(name, B):
+    # PSS_ACCUM_F32: the gradient is a recursive fp32 sum in atomic order, so
+    # element e with n_e contributions may be off by (n_e - 1) u A_e (Higham).
+    w = wl.make_workload(name, B=B)
+    h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_ACCUM, binding.ACCUM_F32)
+    h.forward(*_batch_cuda(w), w.B)
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    ref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
+    A = o.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    n = o.grad(w.indices, w.offsets, w.B, np.ones_like(w.grad_out))
+    bound = np.maximum(n - 1, 1) * gu.U32 * A + gu.U32 * np.abs(ref)
+    assert np.all(np.abs(g.astype(np.float64) - ref) <= bound)
+    # SGD scattered straight into M: same bound on the step, plus the operand rounding
+    h.forward(*_batch_cuda(w), w.B)
+    if w.opt == "sgd":
+        h.backward_update(gu.cuda(w.grad_out), w.lr)
+        w2, _, _ = o.step(w.w0, None, w.indices, w.offsets, w.B, w.grad_out, "sgd", w.lr)
+        err = np.abs(gu.host(h.get_weights()).astype(np.float64) - w2)
+        scale = np.abs(w.w0).astype(np.float64) + w.lr * A
+        assert np.all(err <= np.maximum(n, 1) * gu.U32 * scale + 2 * gu.U32 * np.abs(w2))
+    h.close()
+
+
 # --------------------------------------------------------------------------
 # full sizes of the named workloads (default launch configuration)
 @pytest.mark.parametrize("name", ["tiny", "kaggle", "tb", "multihot", "microbench"])
