@@ -68,7 +68,8 @@ typedef enum {
     PSS_ERR_STATE = 4,         /* call order violated (e.g. backward before forward) */
     PSS_ERR_INDEX_RANGE = 5,   /* the device saw an id outside its table, or bad offsets */
     PSS_ERR_TIMEOUT = 6,       /* a bounded device wait gave up */
-    PSS_ERR_UNSUPPORTED = 7    /* valid request this build does not implement */
+    PSS_ERR_UNSUPPORTED = 7,   /* valid request this build does not implement */
+    PSS_ERR_CAPACITY = 8       /* request exceeds a fixed capacity (pss_grad_noalloc) */
 } pss_status;
 
 typedef enum { PSS_SGD = 0, PSS_ADAGRAD = 1 } pss_optimizer;
@@ -230,6 +231,39 @@ pss_status pss_reset_profile(pss_handle* h);
 
 /* Static description of a status code. */
 const char* pss_status_string(pss_status s);
+
+/*
+ * Gradient of the shared array for one batch WITHOUT ALLOCATING device memory.
+ * (The paper has no counterpart: this is a deployment aid of this library.)
+ * For callers that cannot call cudaMalloc: code embedded in a host framework
+ * that owns the whole device-memory budget and forbids side allocations, and
+ * latency-critical code that cannot accept the implicit device synchronisation
+ * an allocation may cause.  No handle is needed and nothing is allocated: the
+ * caller passes every input and the output, and the fp64 accumulator lives in
+ * a file-scope device array of fixed size, held by every GPU that loads the
+ * library until the process exits.
+ *   Computes, like pss_backward_grad with PSS_ACCUM_F64, for the mapping given
+ *   by (table_cardinalities, num_tables, dim, M, Z, G, seed) as in pss_create:
+ *     grad[e] = sum over every (bag, id, chunk j, z) with loc + z == e of grad_out[b][t][jZ+z]
+ *   table_cardinalities: host, num_tables entries.  indices, offsets, grad_out,
+ *   grad (fp32[M], overwritten) and first_bad: DEVICE memory (host pointers are
+ *   rejected: nothing is staged).  first_bad (optional, int64[1]) receives the
+ *   smallest position of an id outside its table (that id is skipped), -2 for
+ *   malformed offsets, or -1.
+ * Capacity: M <= 4194304 (2^22: 32 MiB of fp64 scratch) and num_tables <= 4096;
+ * larger requests return PSS_ERR_CAPACITY before any device work is queued.
+ * The first call on a device looks up the scratch's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture.  Every call shares the one scratch array: calls whose work overlaps
+ * on the GPU (other streams, other threads) race and give wrong results, so
+ * order them on one stream or synchronise between them.  Asynchronous on
+ * `stream`.  Errors: PSS_ERR_INVALID_ARG, PSS_ERR_CAPACITY, PSS_ERR_CUDA.
+ */
+pss_status pss_grad_noalloc(const int64_t* table_cardinalities, int32_t num_tables, int32_t dim,
+                            int64_t M, int32_t Z, int32_t G, uint64_t seed,
+                            const int64_t* indices, int64_t nnz, const int64_t* offsets,
+                            int64_t B, const float* grad_out, float* grad, int64_t* first_bad,
+                            pss_stream stream);
 
 #ifdef __cplusplus
 }

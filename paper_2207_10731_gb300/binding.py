@@ -20,7 +20,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libpss.so")
 
 PSS_OK, PSS_ERR_INVALID_ARG, PSS_ERR_OOM, PSS_ERR_CUDA, PSS_ERR_STATE, PSS_ERR_INDEX_RANGE, \
-    PSS_ERR_TIMEOUT, PSS_ERR_UNSUPPORTED = range(8)
+    PSS_ERR_TIMEOUT, PSS_ERR_UNSUPPORTED, PSS_ERR_CAPACITY = range(9)
 PSS_SGD, PSS_ADAGRAD = 0, 1
 OPT_BACKWARD_PATH, OPT_UPDATE_MODE, OPT_PROFILE, OPT_SYNC_CHECK, OPT_ACCUM = 1, 2, 3, 4, 5
 ACCUM_F64, ACCUM_F32 = 0, 1
@@ -34,7 +34,7 @@ EXPORTS = [
     "pss_create", "pss_destroy", "pss_set_weights", "pss_get_weights", "pss_get_state",
     "pss_set_state", "pss_compute_locations", "pss_forward", "pss_backward_update",
     "pss_backward_grad", "pss_set_option", "pss_get_option", "pss_get_error", "pss_get_info",
-    "pss_get_profile", "pss_reset_profile", "pss_status_string",
+    "pss_get_profile", "pss_reset_profile", "pss_status_string", "pss_grad_noalloc",
 ]
 
 
@@ -87,6 +87,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "pss_get_info": [vp, vp],
             "pss_get_profile": [vp, i32, vp, vp],
             "pss_reset_profile": [vp],
+            "pss_grad_noalloc": [vp, i32, i32, i64, i32, i32, u64, vp, i64, vp, i64, vp, vp, vp,
+                                 vp],
         }
         for name, args in sigs.items():
             fn = getattr(lib, name)

@@ -248,6 +248,9 @@ const char* pss_status_string(pss_status s) {
         case PSS_ERR_INDEX_RANGE: return "id outside its table, or malformed offsets";
         case PSS_ERR_TIMEOUT: return "device wait timed out";
         case PSS_ERR_UNSUPPORTED: return "unsupported";
+        case PSS_ERR_CAPACITY:
+            return "exceeds the fixed scratch capacity of pss_grad_noalloc (M <= 4194304, "
+                   "tables <= 4096)";
     }
     return "unknown status";
 }

@@ -96,3 +96,8 @@ def check_adagrad(w_gpu, G_gpu, w_ref, G_ref, g_ref, A, lr, tol=GRAD_TOL, what="
     badw = errw > boundw
     assert not badw.any(), (f"{what}: weights off at {int(badw.sum())} elements; worst err "
                             f"{errw[badw].max():.3e}")
+
+
+def ctypes_ptr(t):
+    import ctypes
+    return ctypes.c_void_p(int(t.data_ptr()))
