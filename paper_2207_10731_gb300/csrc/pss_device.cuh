@@ -61,4 +61,138 @@ __device__ __forceinline__ void kahan_add(float& s, float& c, float x) {
     s = t;
 }
 
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+
+inline int ceil_log2(int v) {
+    int l = 0;
+    while ((1 << l) < v) ++l;
+    return l;
+}
+
+// Grid of a grid-stride kernel: all CTAs that fit at once, capped by the work.
+template <typename K>
+int grid_for(K kernel, int sm_count, int64_t work_blocks, size_t smem = 0) {
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kThreads, smem) !=
+            cudaSuccess ||
+        per_sm < 1)
+        per_sm = 1;
+    int64_t g = (int64_t)sm_count * per_sm;
+    if (work_blocks < g) g = work_blocks;
+    if (g < 1) g = 1;
+    return (int)g;
+}
+
+// Per-lane column description inside one bag row.
+template <int VW, int KC>
+struct Cols {
+    int j[KC];     // chunk of the column
+    int z[KC];     // offset of the column inside its chunk
+    bool v[KC];    // column exists (d not a multiple of the group width)
+    int e[KC];     // element offset of the column in the row
+    __device__ __forceinline__ Cols(const DevParams& p, int lg, int gs) {
+        const int V = p.d / VW;
+#pragma unroll
+        for (int k = 0; k < KC; ++k) {
+            const int c = lg + k * gs;
+            v[k] = c < V;
+            e[k] = c * VW;
+            j[k] = e[k] / p.Z;
+            z[k] = e[k] - j[k] * p.Z;
+        }
+    }
+};
+
+template <int VW>
+struct Vec;
+template <>
+struct Vec<4> {
+    using T = float4;
+    static __device__ __forceinline__ float4 ldg(const float* p) {
+        return __ldg(reinterpret_cast<const float4*>(p));
+    }
+    static __device__ __forceinline__ float4 ldcs(const float* p) {
+        return __ldcs(reinterpret_cast<const float4*>(p));
+    }
+    static __device__ __forceinline__ void stcs(float* p, float4 v) {
+        __stcs(reinterpret_cast<float4*>(p), v);
+    }
+    static __device__ __forceinline__ void red(float* p, float4 v) { red_add_v4(p, v); }
+    static __device__ __forceinline__ float get(const float4& v, int i) {
+        return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+    }
+    static __device__ __forceinline__ void set(float4& v, int i, float x) {
+        if (i == 0) v.x = x; else if (i == 1) v.y = x; else if (i == 2) v.z = x; else v.w = x;
+    }
+    static __device__ __forceinline__ float4 scale(float4 v, float s) {
+        return make_float4(__fmul_rn(v.x, s), __fmul_rn(v.y, s), __fmul_rn(v.z, s),
+                           __fmul_rn(v.w, s));
+    }
+};
+template <>
+struct Vec<1> {
+    using T = float;
+    static __device__ __forceinline__ float ldg(const float* p) { return __ldg(p); }
+    static __device__ __forceinline__ float ldcs(const float* p) { return __ldcs(p); }
+    static __device__ __forceinline__ void stcs(float* p, float v) { __stcs(p, v); }
+    static __device__ __forceinline__ void red(float* p, float v) { red_add_f32(p, v); }
+    static __device__ __forceinline__ float get(const float& v, int) { return v; }
+    static __device__ __forceinline__ void set(float& v, int, float x) { v = x; }
+    static __device__ __forceinline__ float scale(float v, float s) { return __fmul_rn(v, s); }
+};
+
+// Bag slot s -> (table t, row b) for s = t*B + b, with Binv = floor((2^64-1)/B):
+// umulhi(s, Binv) is t or t-1 (same argument as the hash's "mod R").
+__device__ __forceinline__ void split_slot(int64_t s, int64_t B, uint64_t Binv, int& t, int64_t& b) {
+    uint64_t q = __umul64hi((uint64_t)s, Binv);
+    uint64_t r = (uint64_t)s - q * (uint64_t)B;
+    if (r >= (uint64_t)B) {
+        ++q;
+        r -= (uint64_t)B;
+    }
+    t = (int)q;
+    b = (int64_t)r;
+}
+
+// Reduction of one VW-wide column into an fp32 or fp64 accumulator.
+template <int VW, typename AT>
+struct Acc;
+template <int VW>
+struct Acc<VW, float> {
+    static __device__ __forceinline__ void red(float* p, typename Vec<VW>::T v) { Vec<VW>::red(p, v); }
+};
+template <>
+struct Acc<1, double> {
+    static __device__ __forceinline__ void red(double* p, float v) { red_add_f64(p, (double)v); }
+};
+
+// Accumulator element -> fp32 gradient (rounded once, to nearest).
+__device__ __forceinline__ float to_f32(float v) { return v; }
+__device__ __forceinline__ float to_f32(double v) { return __double2float_rn(v); }
+
+__device__ __forceinline__ bool bag_range(const int64_t* __restrict__ off, int64_t s, int64_t nnz,
+                                          int64_t& q0, int64_t& q1) {
+    q0 = __ldg(off + s);
+    q1 = __ldg(off + s + 1);
+    if (q0 < 0 || q1 < q0 || q1 > nnz) {
+        q0 = q1 = 0;
+        return false;
+    }
+    return true;
+}
+
+
+// Record a distinct block start x in the touched bitmap / list (first marker appends).
+__device__ __forceinline__ void mark_touched(const Touched& tc, uint64_t x) {
+    uint32_t* wp = tc.bitmap + (x >> 5);
+    const uint32_t bit = 1u << (x & 31);
+    if (*reinterpret_cast<volatile uint32_t*>(wp) & bit) return;
+    const uint32_t old = atomicOr(wp, bit);
+    if (!(old & bit)) {
+        const unsigned long long slot = atomicAdd(tc.count, 1ULL);
+        if ((int64_t)slot < tc.cap) tc.list[slot] = (int64_t)x;
+    }
+}
+
 }  // namespace pss

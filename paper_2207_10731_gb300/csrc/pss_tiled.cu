@@ -1,0 +1,448 @@
+// Tiled forward (hash + gather + sum-pool) and backward scatter kernels.
+//
+// A CTA takes a TILE of `tb` consecutive bags of one table (bag slots
+// t*B + b0 .. t*B + b0 + tb - 1, so the table id is uniform in the tile):
+//   stage:  the tile's offsets go to shared memory; then every (id, chunk)
+//           pair of the tile is hashed ONCE, by one thread, into a shared
+//           array of block buckets x (loc = G*x).  Long tiles are staged in
+//           chunks of `qc` ids.
+//   gather / scatter: groups of gs lanes own consecutive bags of the tile and
+//           walk their ids in order, U ids at a time so that U independent
+//           16-byte loads per lane are in flight; a bag's row is stored when
+//           its last id has been added (empty bags store zeros).
+// Everything is index arithmetic on the CSR batch; no sort, no atomics in the
+// forward.  The backward adds each bag's upstream-gradient row into every
+// block the bag read (the dense branch of Algorithm 1) with global reductions:
+// 16-byte fp32 vector reductions, or one fp64 reduction per element with
+// consecutive lanes on consecutive elements (8 sectors per instruction).
+#include <climits>
+
+#include "pss_device.cuh"
+#include "pss_internal.h"
+
+namespace pss {
+namespace {
+
+constexpr int kU = 4;            // ids in flight per group
+constexpr int kBagsPerGroup = 16;
+
+template <typename XT>
+struct Invalid;
+template <>
+struct Invalid<uint32_t> {
+    static constexpr uint32_t v = 0xffffffffu;
+};
+template <>
+struct Invalid<uint64_t> {
+    static constexpr uint64_t v = ~uint64_t(0);
+};
+
+struct TileGeom {
+    int tb;               // bags per tile
+    int qc;               // ids per staging chunk
+    int tiles_per_table;  // ceil(B / tb)
+};
+
+// Stage the offsets of tile (t, b0) into s_off; returns false (and zeroes the
+// tile's rows when `out` is given) if the offsets are malformed.
+__device__ __forceinline__ bool stage_offsets(const int64_t* __restrict__ off, int64_t s0, int nb,
+                                              int64_t nnz, int64_t* s_off, int* s_bad,
+                                              DevError* err) {
+    if (threadIdx.x == 0) *s_bad = 0;
+    for (int i = threadIdx.x; i <= nb; i += kThreads) s_off[i] = __ldg(off + s0 + i);
+    __syncthreads();
+    for (int i = threadIdx.x; i < nb; i += kThreads) {
+        const int64_t a = s_off[i], c = s_off[i + 1];
+        if (a < 0 || c < a || c > nnz) *s_bad = 1;
+    }
+    __syncthreads();
+    const bool bad = *s_bad != 0;
+    if (bad && threadIdx.x == 0) record_bad_offsets(err);
+    return !bad;
+}
+
+// Hash every (id, chunk) pair of ids [qc0, qc0 + nq) of table t into s_x.
+template <typename XT, bool TOUCH>
+__device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t* __restrict__ idx,
+                                              int t, uint64_t card, int64_t qc0, int nq, XT* s_x,
+                                              DevError* err, const Touched& tc) {
+    const int npairs = nq * p.J;
+    for (int k = threadIdx.x; k < npairs; k += kThreads) {
+        const int qi = k / p.J;
+        const int j = k - qi * p.J;
+        const int64_t q = qc0 + qi;
+        const int64_t id = __ldg(idx + q);
+        XT x;
+        if ((uint64_t)id >= card) {
+            x = Invalid<XT>::v;
+            if (j == 0) record_bad_id(err, q);
+        } else {
+            const uint64_t b = hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
+            x = (XT)b;
+            if (TOUCH) mark_touched(tc, b);
+        }
+        s_x[k] = x;
+    }
+}
+
+// ---------------------------------------------------------------------------
+template <int VW, int KC, typename XT>
+__global__ void __launch_bounds__(kThreads)
+k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
+                const int64_t* __restrict__ off, int64_t B, const float* __restrict__ w,
+                float* __restrict__ out, DevError* err, int log2gs, TileGeom tg) {
+    using V = Vec<VW>;
+    using VT = typename V::T;
+    extern __shared__ __align__(16) unsigned char smem[];
+    int64_t* s_off = reinterpret_cast<int64_t*>(smem);
+    XT* s_x = reinterpret_cast<XT*>(s_off + tg.tb + 1);
+    __shared__ int s_bad;
+
+    const int lane = threadIdx.x & 31;
+    const int gs = 1 << log2gs;
+    const int lg = lane & (gs - 1);
+    const int grp = (threadIdx.x >> 5) * (32 >> log2gs) + (lane >> log2gs);
+    const Cols<VW, KC> col(p, lg, gs);
+    const uint64_t G = (uint64_t)p.G;
+    const int J = p.J;
+    const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
+    const Touched none{};
+
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int t = (int)(tile / tg.tiles_per_table);
+        const int64_t b0 = (tile - (int64_t)t * tg.tiles_per_table) * tg.tb;
+        const int nb = (int)((B - b0) < tg.tb ? (B - b0) : tg.tb);
+        const int64_t s0 = (int64_t)t * B + b0;
+        const int gb0 = min(grp * kBagsPerGroup, nb);
+        const int gb1 = min(gb0 + kBagsPerGroup, nb);
+        float* obase = out + ((b0 * p.T) + t) * (int64_t)p.d;   // row of bag b0
+        const int64_t ostride = (int64_t)p.T * p.d;               // next bag row
+
+        if (!stage_offsets(off, s0, nb, nnz, s_off, &s_bad, err)) {
+            for (int bi = gb0; bi < gb1; ++bi)
+#pragma unroll
+                for (int k = 0; k < KC; ++k) {
+                    if (!col.v[k]) continue;
+                    VT z;
+#pragma unroll
+                    for (int i = 0; i < VW; ++i) V::set(z, i, 0.f);
+                    V::stcs(obase + bi * ostride + col.e[k], z);
+                }
+            __syncthreads();
+            continue;
+        }
+        const uint64_t card = (uint64_t)__ldg(p.cards + t);
+        const int64_t qa = s_off[0], qb = s_off[nb];
+        const int64_t gq0 = s_off[gb0], gq1 = s_off[gb1];
+        int bi = gb0;
+        int64_t qend = (gb0 < gb1) ? s_off[gb0 + 1] : 0;
+        float acc[KC][VW], cmp[KC][VW];
+#pragma unroll
+        for (int k = 0; k < KC; ++k)
+#pragma unroll
+            for (int i = 0; i < VW; ++i) acc[k][i] = cmp[k][i] = 0.f;
+
+        auto flush = [&]() {
+            float* orow = obase + bi * ostride;
+#pragma unroll
+            for (int k = 0; k < KC; ++k) {
+                if (!col.v[k]) continue;
+                VT o;
+#pragma unroll
+                for (int i = 0; i < VW; ++i) {
+                    V::set(o, i, acc[k][i]);
+                    acc[k][i] = cmp[k][i] = 0.f;
+                }
+                V::stcs(orow + col.e[k], o);
+            }
+        };
+
+        for (int64_t qc0 = qa; qc0 < qb; qc0 += tg.qc) {
+            const int nq = (int)((qb - qc0) < tg.qc ? (qb - qc0) : tg.qc);
+            stage_buckets<XT, false>(p, idx, t, card, qc0, nq, s_x, err, none);
+            __syncthreads();
+            const int64_t qlo = gq0 > qc0 ? gq0 : qc0;
+            const int64_t qhi = gq1 < qc0 + nq ? gq1 : qc0 + nq;
+            for (int64_t q = qlo; q < qhi; q += kU) {
+                VT v[kU][KC];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+#pragma unroll
+                    for (int k = 0; k < KC; ++k) {
+#pragma unroll
+                        for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
+                        if (q + u < qhi && col.v[k]) {
+                            const XT x = s_x[(int)(q + u - qc0) * J + col.j[k]];
+                            if (x != Invalid<XT>::v) v[u][k] = V::ldg(w + G * (uint64_t)x + col.z[k]);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    if (q + u >= qhi) break;
+                    while (q + u >= qend) {
+                        flush();
+                        ++bi;
+                        qend = s_off[bi + 1];
+                    }
+#pragma unroll
+                    for (int k = 0; k < KC; ++k)
+#pragma unroll
+                        for (int i = 0; i < VW; ++i) kahan_add(acc[k][i], cmp[k][i], V::get(v[u][k], i));
+                }
+            }
+            __syncthreads();
+        }
+        // the current bag and any trailing empty bags
+        while (bi < gb1) {
+            flush();
+            ++bi;
+        }
+        __syncthreads();
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Backward scatter: target[G*x + z] += scale * grad_out row chunk.
+template <int VW, int KC, typename XT, typename AT, bool TOUCH>
+__global__ void __launch_bounds__(kThreads)
+k_scatter_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
+                const int64_t* __restrict__ off, int64_t B, const float* __restrict__ gout,
+                float scale, AT* __restrict__ target, Touched tc, DevError* err, int log2gs,
+                TileGeom tg) {
+    using V = Vec<VW>;
+    using VT = typename V::T;
+    extern __shared__ __align__(16) unsigned char smem[];
+    int64_t* s_off = reinterpret_cast<int64_t*>(smem);
+    XT* s_x = reinterpret_cast<XT*>(s_off + tg.tb + 1);
+    __shared__ int s_bad;
+
+    const int lane = threadIdx.x & 31;
+    const int gs = 1 << log2gs;
+    const int lg = lane & (gs - 1);
+    const int grp = (threadIdx.x >> 5) * (32 >> log2gs) + (lane >> log2gs);
+    const Cols<VW, KC> col(p, lg, gs);
+    const uint64_t G = (uint64_t)p.G;
+    const int J = p.J;
+    const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
+
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        const int t = (int)(tile / tg.tiles_per_table);
+        const int64_t b0 = (tile - (int64_t)t * tg.tiles_per_table) * tg.tb;
+        const int nb = (int)((B - b0) < tg.tb ? (B - b0) : tg.tb);
+        const int64_t s0 = (int64_t)t * B + b0;
+        const int gb0 = min(grp * kBagsPerGroup, nb);
+        const int gb1 = min(gb0 + kBagsPerGroup, nb);
+        const float* gbase = gout + ((b0 * p.T) + t) * (int64_t)p.d;
+        const int64_t gstride = (int64_t)p.T * p.d;
+
+        if (!stage_offsets(off, s0, nb, nnz, s_off, &s_bad, err)) {
+            __syncthreads();
+            continue;
+        }
+        const uint64_t card = (uint64_t)__ldg(p.cards + t);
+        const int64_t qa = s_off[0], qb = s_off[nb];
+        const int64_t gq0 = s_off[gb0], gq1 = s_off[gb1];
+        int bi = gb0;                       // bag of the next id
+        int64_t qend = (gb0 < gb1) ? s_off[gb0 + 1] : 0;
+        int have = -1;                      // bag whose row is in `row`
+        VT row[KC];
+
+        for (int64_t qc0 = qa; qc0 < qb; qc0 += tg.qc) {
+            const int nq = (int)((qb - qc0) < tg.qc ? (qb - qc0) : tg.qc);
+            stage_buckets<XT, TOUCH>(p, idx, t, card, qc0, nq, s_x, err, tc);
+            __syncthreads();
+            const int64_t qlo = gq0 > qc0 ? gq0 : qc0;
+            const int64_t qhi = gq1 < qc0 + nq ? gq1 : qc0 + nq;
+            for (int64_t q = qlo; q < qhi; q += kU) {
+                // bags of the next kU ids, and their rows (independent loads)
+                int ub[kU];
+                VT r[kU][KC];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    ub[u] = -1;
+                    if (q + u < qhi) {
+                        while (q + u >= qend) {
+                            ++bi;
+                            qend = s_off[bi + 1];
+                        }
+                        ub[u] = bi;
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    if (ub[u] < 0) continue;
+                    const bool same_prev = (u > 0) ? (ub[u] == ub[u - 1]) : (ub[u] == have);
+                    if (same_prev) continue;
+#pragma unroll
+                    for (int k = 0; k < KC; ++k)
+                        if (col.v[k])
+                            r[u][k] = V::scale(V::ldcs(gbase + ub[u] * gstride + col.e[k]), scale);
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    if (ub[u] < 0) break;
+                    const bool same_prev = (u > 0) ? (ub[u] == ub[u - 1]) : (ub[u] == have);
+                    if (!same_prev) {
+#pragma unroll
+                        for (int k = 0; k < KC; ++k) row[k] = r[u][k];
+                        have = ub[u];
+                    }
+#pragma unroll
+                    for (int k = 0; k < KC; ++k) {
+                        if (!col.v[k]) continue;
+                        const XT x = s_x[(int)(q + u - qc0) * J + col.j[k]];
+                        if (x != Invalid<XT>::v)
+                            Acc<VW, AT>::red(target + G * (uint64_t)x + col.z[k], row[k]);
+                    }
+                }
+            }
+            __syncthreads();
+        }
+        __syncthreads();
+    }
+}
+
+TileGeom tile_geom(const DevParams& p, const RowLayout& lay, int64_t B, size_t xbytes) {
+    TileGeom g;
+    const int ng = 32 >> lay.log2gs;
+    g.tb = kWarps * ng * kBagsPerGroup;
+    const int stage_bytes = 16384;
+    g.qc = stage_bytes / (int)(xbytes * (size_t)p.J);
+    if (g.qc < 1) g.qc = 1;
+    g.tiles_per_table = (int)((B + g.tb - 1) / g.tb);
+    return g;
+}
+
+size_t tile_smem(const TileGeom& g, const DevParams& p, size_t xbytes) {
+    return sizeof(int64_t) * (size_t)(g.tb + 1) + xbytes * (size_t)g.qc * (size_t)p.J;
+}
+
+template <int VW, int KC, typename XT>
+cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
+                     const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
+                     int sm_count, cudaStream_t st) {
+    const TileGeom tg = tile_geom(p, lay, B, sizeof(XT));
+    const size_t smem = tile_smem(tg, p, sizeof(XT));
+    const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
+    const int grid = grid_for(k_forward_tiled<VW, KC, XT>, sm_count, ntiles, smem);
+    k_forward_tiled<VW, KC, XT><<<grid, kThreads, smem, st>>>(p, idx, nnz, off, B, w, out, err,
+                                                              lay.log2gs, tg);
+    return cudaGetLastError();
+}
+
+template <int VW, int KC, typename XT, typename AT, bool TOUCH>
+cudaError_t sc_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
+                    const int64_t* off, int64_t B, const float* gout, float scale, AT* target,
+                    const Touched& tc, DevError* err, int sm_count, cudaStream_t st) {
+    const TileGeom tg = tile_geom(p, lay, B, sizeof(XT));
+    const size_t smem = tile_smem(tg, p, sizeof(XT));
+    const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
+    const int grid = grid_for(k_scatter_tiled<VW, KC, XT, AT, TOUCH>, sm_count, ntiles, smem);
+    k_scatter_tiled<VW, KC, XT, AT, TOUCH><<<grid, kThreads, smem, st>>>(
+        p, idx, nnz, off, B, gout, scale, target, tc, err, lay.log2gs, tg);
+    return cudaGetLastError();
+}
+
+template <int VW, int KC>
+cudaError_t fwd_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
+                  const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
+                  int sm_count, cudaStream_t st) {
+    if (p.R < 0xffffffffull)
+        return fwd_inst<VW, KC, uint32_t>(p, lay, idx, nnz, off, B, w, out, err, sm_count, st);
+    return fwd_inst<VW, KC, uint64_t>(p, lay, idx, nnz, off, B, w, out, err, sm_count, st);
+}
+
+template <int VW, int KC, typename AT>
+cudaError_t sc_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
+                 const int64_t* off, int64_t B, const float* gout, float scale, AT* target,
+                 const Touched* tc, DevError* err, int sm_count, cudaStream_t st) {
+    const Touched none{};
+    const bool wide = p.R >= 0xffffffffull;
+    if (tc) {
+        if (wide)
+            return sc_inst<VW, KC, uint64_t, AT, true>(p, lay, idx, nnz, off, B, gout, scale, target,
+                                                        *tc, err, sm_count, st);
+        return sc_inst<VW, KC, uint32_t, AT, true>(p, lay, idx, nnz, off, B, gout, scale, target,
+                                                    *tc, err, sm_count, st);
+    }
+    if (wide)
+        return sc_inst<VW, KC, uint64_t, AT, false>(p, lay, idx, nnz, off, B, gout, scale, target,
+                                                     none, err, sm_count, st);
+    return sc_inst<VW, KC, uint32_t, AT, false>(p, lay, idx, nnz, off, B, gout, scale, target, none,
+                                                 err, sm_count, st);
+}
+
+}  // namespace
+
+cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
+                           int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
+                           DevError* err, int sm_count, cudaStream_t st) {
+#define PSS_FW(VW, KC) return fwd_x<VW, KC>(p, lay, idx, nnz, off, B, w, out, err, sm_count, st)
+    if (lay.vw == 4) {
+        switch (lay.kc) {
+            case 1: PSS_FW(4, 1);
+            case 2: PSS_FW(4, 2);
+            case 4: PSS_FW(4, 4);
+        }
+    } else {
+        switch (lay.kc) {
+            case 1: PSS_FW(1, 1);
+            case 2: PSS_FW(1, 2);
+            case 4: PSS_FW(1, 4);
+            case 8: PSS_FW(1, 8);
+            case 16: PSS_FW(1, 16);
+        }
+    }
+#undef PSS_FW
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_scatter(const DevParams& p, const RowLayout& lay, const int64_t* idx,
+                           int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
+                           float scale, float* target, const Touched* touched, DevError* err,
+                           int sm_count, cudaStream_t st) {
+#define PSS_SC(VW, KC) \
+    return sc_x<VW, KC, float>(p, lay, idx, nnz, off, B, grad_out, scale, target, touched, err, \
+                               sm_count, st)
+    if (lay.vw == 4) {
+        switch (lay.kc) {
+            case 1: PSS_SC(4, 1);
+            case 2: PSS_SC(4, 2);
+            case 4: PSS_SC(4, 4);
+        }
+    } else {
+        switch (lay.kc) {
+            case 1: PSS_SC(1, 1);
+            case 2: PSS_SC(1, 2);
+            case 4: PSS_SC(1, 4);
+            case 8: PSS_SC(1, 8);
+            case 16: PSS_SC(1, 16);
+        }
+    }
+#undef PSS_SC
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_scatter64(const DevParams& p, const RowLayout& lay_in, const int64_t* idx,
+                             int64_t nnz, const int64_t* off, int64_t B, const float* grad_out,
+                             double* target, const Touched* touched, DevError* err, int sm_count,
+                             cudaStream_t st) {
+    // fp64 reductions are scalar: lanes on consecutive elements
+    const RowLayout lay = choose_layout(p.d, 1, 1);
+    (void)lay_in;
+#define PSS_SC(KC) \
+    return sc_x<1, KC, double>(p, lay, idx, nnz, off, B, grad_out, 1.0f, target, touched, err, \
+                               sm_count, st)
+    switch (lay.kc) {
+        case 1: PSS_SC(1);
+        case 2: PSS_SC(2);
+        case 4: PSS_SC(4);
+        case 8: PSS_SC(8);
+        case 16: PSS_SC(16);
+    }
+#undef PSS_SC
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace pss
