@@ -278,6 +278,8 @@ def run_gpu(args):
         h.set_weights(base.repeat(-(-w.M // base.numel()))[: w.M].contiguous())
         del base
     h.set_option(binding.OPT_ACCUM, binding.ACCUM_F32 if args.accum == "f32" else binding.ACCUM_F64)
+    h.set_option(binding.OPT_BACKWARD_PATH, {"auto": binding.PATH_AUTO, "atomic": binding.PATH_ATOMIC,
+                                             "sorted": binding.PATH_SORTED}[args.path])
     out = torch.empty((w.B, w.T, w.d), dtype=torch.float32, device=dev)
     nnz_per_step = [int(b[0].shape[0]) for b in batches]
     stream = torch.cuda.current_stream()
@@ -389,6 +391,7 @@ def run_gpu(args):
                        "seq_len": 1,
                        "parallelism": "independent replicas" if world > 1 else "single GPU",
                        "grad_accumulator": args.accum,
+                       "backward_path": ["auto", "atomic", "sorted"][h.info()["last_path"]],
                        "l2": (f"inputs larger than L2: {args.rotate}-batch rotation, "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB output and "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB upstream gradient per step")},
@@ -430,6 +433,8 @@ def main(argv=None):
     ap.add_argument("--accum", choices=["f64", "f32"], default="f64",
                     help="gradient accumulator precision of the atomic path")
     ap.add_argument("--B", type=int, default=None, help="override the batch size (profiling)")
+    ap.add_argument("--path", choices=["auto", "atomic", "sorted"], default="auto",
+                    help="backward path")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")

@@ -73,6 +73,15 @@ struct pss_handle {
     Touched touched{};
     int64_t touched_words = 0;
 
+    // sorted backward path (allocated on first use)
+    SortedBuffers sb{};
+    int64_t sb_pairs_cap = 0, sb_ids_cap = 0;
+    bool sb_counters = false;
+    bool batch_emitted = false;                 // the last forward wrote pair_x / q_row
+    unsigned long long* stats_host = nullptr;   // pinned mirror of sb.stats
+    cudaEvent_t stats_ev = nullptr;
+    bool stats_pending = false;
+
     // profiling
     std::vector<EventPair> ev[PSS_K_COUNT];
     std::vector<EventPair> ev_free;
@@ -142,21 +151,23 @@ EventPair take_events(pss_handle* h) {
     return e;
 }
 
-// Bracket one launch: counts it and, when profiling, records events on its stream.
+// Bracket n launches of one kernel kind: counts them and, when profiling,
+// records events on their stream.
 struct LaunchScope {
     pss_handle* h;
     int k;
     cudaStream_t st;
+    int n;
     EventPair ev{nullptr, nullptr};
-    LaunchScope(pss_handle* h_, int k_, cudaStream_t st_) : h(h_), k(k_), st(st_) {
+    LaunchScope(pss_handle* h_, int k_, cudaStream_t st_, int n_ = 1) : h(h_), k(k_), st(st_), n(n_) {
         if (h->profile) {
             ev = take_events(h);
             cudaEventRecord(ev.a, st);
         }
     }
     ~LaunchScope() {
-        h->launches++;
-        h->launches_by_kernel[k]++;
+        h->launches += n;
+        h->launches_by_kernel[k] += n;
         if (h->profile && ev.a) {
             cudaEventRecord(ev.b, st);
             h->ev[k].push_back(ev);
@@ -218,6 +229,76 @@ bool use_touched(const pss_handle* h, int64_t pairs) {
     // dense pass reads/writes ~5 words per element of M; the touched pass
     // costs ~5 words per element of each distinct block plus the marking.
     return h->dp.M > 2 * pairs * (int64_t)h->dp.L;
+}
+
+// Largest bucket count for which the sorted path keeps per-bucket counters
+// (4 bytes each, twice); AUTO takes the sorted path up to kAutoSortedMaxR.
+constexpr int64_t kSortedMaxR = int64_t(1) << 28;
+constexpr int64_t kAutoSortedMaxR = int64_t(1) << 26;
+
+bool sorted_supported(const pss_handle* h, int64_t nnz, int64_t B) {
+    const int64_t J = h->dp.J;
+    return (int64_t)h->dp.R <= kSortedMaxR && nnz * J < (int64_t)0xffffffffLL &&
+           (int64_t)h->dp.T * B * J < (int64_t)0xffffffffLL;
+}
+
+bool want_sorted(const pss_handle* h) {
+    if (h->path == PSS_PATH_SORTED) return true;
+    if (h->path == PSS_PATH_ATOMIC) return false;
+    return (int64_t)h->dp.R <= kAutoSortedMaxR;
+}
+
+pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {
+    const int64_t R = (int64_t)h->dp.R;
+    const int64_t npairs = nnz * h->dp.J;
+    if (!h->sb_counters) {
+        const int64_t nblk = sorted_scan_blocks(R);
+        PSS_TRY(cudaMalloc(&h->sb.cnt, sizeof(uint32_t) * (size_t)R));
+        PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)R, st));
+        PSS_TRY(cudaMalloc(&h->sb.start, sizeof(uint32_t) * (size_t)(R + 1)));
+        PSS_TRY(cudaMalloc(&h->sb.bsum, sizeof(uint32_t) * (size_t)nblk));
+        PSS_TRY(cudaMalloc(&h->sb.btask, sizeof(uint32_t) * (size_t)nblk));
+        PSS_TRY(cudaMalloc(&h->sb.bnz, sizeof(uint32_t) * (size_t)nblk));
+        PSS_TRY(cudaMalloc(&h->sb.stats, 3 * sizeof(unsigned long long)));
+        PSS_TRY(cudaMemsetAsync(h->sb.stats, 0, 3 * sizeof(unsigned long long), st));
+        PSS_TRY(cudaMallocHost(&h->stats_host, 2 * sizeof(unsigned long long)));
+        h->stats_host[0] = h->stats_host[1] = 0;
+        PSS_TRY(cudaEventCreateWithFlags(&h->stats_ev, cudaEventDisableTiming));
+        h->sb_counters = true;
+    }
+    if (h->sb_pairs_cap < npairs) {
+        for (uint32_t** b : {&h->sb.pair_x, &h->sb.sorted_r}) {
+            if (*b) PSS_TRY(cudaFreeAsync(*b, st));
+            *b = nullptr;
+        }
+        if (h->sb.tasks) PSS_TRY(cudaFreeAsync(h->sb.tasks, st));
+        h->sb.tasks = nullptr;
+        h->sb_pairs_cap = 0;
+        const size_t bytes = sizeof(uint32_t) * (size_t)(npairs > 0 ? npairs : 1);
+        PSS_TRY(cudaMallocAsync(&h->sb.pair_x, bytes, st));
+        PSS_TRY(cudaMallocAsync(&h->sb.sorted_r, bytes, st));
+        PSS_TRY(cudaMallocAsync(&h->sb.tasks,
+                                sizeof(uint2) * (size_t)sorted_max_tasks(R, npairs), st));
+        h->sb_pairs_cap = npairs;
+    }
+    if (h->sb_ids_cap < nnz) {
+        if (h->sb.q_row) PSS_TRY(cudaFreeAsync(h->sb.q_row, st));
+        h->sb.q_row = nullptr;
+        h->sb_ids_cap = 0;
+        PSS_TRY(cudaMallocAsync(&h->sb.q_row, sizeof(uint32_t) * (size_t)(nnz > 0 ? nnz : 1), st));
+        h->sb_ids_cap = nnz;
+    }
+    return PSS_OK;
+}
+
+// Collision rate of the last sorted pass, once its statistics have arrived.
+void poll_stats(pss_handle* h) {
+    if (h->stats_pending && cudaEventQuery(h->stats_ev) == cudaSuccess) {
+        const double pairs = (double)h->stats_host[0];
+        h->last_collision = pairs > 0 ? 1.0 - (double)h->stats_host[1] / pairs : 0.0;
+        h->stats_pending = false;
+    }
+    cudaGetLastError();
 }
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -351,6 +432,12 @@ pss_status pss_destroy(pss_handle* h) {
     cudaFree(h->touched.bitmap);
     cudaFree(h->touched.list);
     cudaFree(h->touched.count);
+    for (void* b : {(void*)h->sb.pair_x, (void*)h->sb.q_row, (void*)h->sb.cnt, (void*)h->sb.start,
+                    (void*)h->sb.bsum, (void*)h->sb.btask, (void*)h->sb.bnz, (void*)h->sb.stats,
+                    (void*)h->sb.tasks, (void*)h->sb.sorted_r})
+        if (b) cudaFree(b);
+    if (h->stats_host) cudaFreeHost(h->stats_host);
+    if (h->stats_ev) cudaEventDestroy(h->stats_ev);
     for (Staging* s : {&h->st_idx, &h->st_off, &h->st_out, &h->st_grad, &h->st_locs})
         if (s->ptr) cudaFree(s->ptr);
     for (int k = 0; k < PSS_K_COUNT; ++k)
@@ -453,11 +540,18 @@ pss_status pss_forward(pss_handle* h, const int64_t* indices, int64_t nnz, const
         PSS_TRY(ensure(h->st_out, nout * sizeof(float), st));
         dout = static_cast<float*>(h->st_out.ptr);
     }
+    const bool emit = nbags > 0 && want_sorted(h) && sorted_supported(h, nnz, B);
+    if (emit) {
+        if ((rc = ensure_sorted(h, nnz, st)) != PSS_OK) return rc;
+        PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)h->dp.R, st));
+    }
     if (nbags > 0) {
         LaunchScope ls(h, PSS_K_FORWARD, st);
         PSS_TRY(launch_forward(h->dp, layout_for(h, dout), di, nnz, doff, B, h->w, dout, h->err,
-                               h->sm_count, st));
+                               emit ? h->sb.pair_x : nullptr, emit ? h->sb.q_row : nullptr,
+                               emit ? h->sb.cnt : nullptr, h->sm_count, st));
     }
+    h->batch_emitted = emit;
     if (host_out)
         PSS_TRY(cudaMemcpyAsync(out, dout, nout * sizeof(float), cudaMemcpyDeviceToHost, st));
     h->last_idx = di;
@@ -491,6 +585,28 @@ static pss_status scatter_into(pss_handle* h, const float* dgrad, float scale, f
                                       touch ? &h->touched : nullptr, h->err, h->sm_count, st));
 }
 
+// Sorted path: histogram, scan, scatter by bucket, segmented reduce into g64.
+static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool touch, cudaStream_t st) {
+    const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
+    if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
+    poll_stats(h);
+    {
+        LaunchScope ls(h, PSS_K_SORT, st, 4);
+        PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, st));
+        PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->sm_count, st));
+    }
+    if (!h->stats_pending) {
+        PSS_TRY(cudaMemcpyAsync(h->stats_host, h->sb.stats, 2 * sizeof(unsigned long long),
+                                cudaMemcpyDeviceToHost, st));
+        PSS_TRY(cudaEventRecord(h->stats_ev, st));
+        h->stats_pending = true;
+    }
+    LaunchScope ls(h, PSS_K_REDUCE, st);
+    PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64,
+                                 touch ? &h->touched : nullptr, h->sm_count, st));
+    return PSS_OK;
+}
+
 pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, pss_stream stream) {
     if (!h) return PSS_ERR_INVALID_ARG;
     if (!h->have_batch) return PSS_ERR_STATE;
@@ -503,8 +619,31 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
     if (rc != PSS_OK) return rc;
     const int64_t pairs = h->last_nnz * (int64_t)h->dp.J;
     const bool ada = h->opt == PSS_ADAGRAD;
-    h->last_path = PSS_PATH_ATOMIC;
-    if (h->accum == PSS_ACCUM_F32 && !ada) {
+    const bool sorted = h->batch_emitted && want_sorted(h);
+    h->last_path = sorted ? PSS_PATH_SORTED : PSS_PATH_ATOMIC;
+    if (sorted) {
+        const int64_t saved = h->accum;
+        h->accum = PSS_ACCUM_F64;                 // the sorted path sums into g64
+        rc = ensure_grad(h, st);
+        h->accum = saved;
+        if (rc != PSS_OK) return rc;
+        const bool touch = use_touched(h, pairs);
+        if (touch && (rc = ensure_touched(h, pairs, st)) != PSS_OK) return rc;
+        if ((rc = sorted_into64(h, dg, touch, st)) != PSS_OK) return rc;
+        {
+            LaunchScope ls(h, PSS_K_UPDATE, st);
+            if (touch)
+                PSS_TRY(launch_update_touched64(ada, h->w, h->Gacc, h->g64, h->touched, h->dp.G,
+                                                h->dp.L, lr, h->eps, h->sm_count, st));
+            else
+                PSS_TRY(launch_update_dense64(ada, h->w, h->Gacc, h->g64, h->dp.M, lr, h->eps,
+                                              h->sm_count, st));
+        }
+        if (touch) {
+            LaunchScope ls(h, PSS_K_MISC, st);
+            PSS_TRY(launch_touched_clear(h->touched, h->sm_count, st));
+        }
+    } else if (h->accum == PSS_ACCUM_F32 && !ada) {
         // SGD is linear in g: scatter -lr * grad_out straight into M.
         if (lr != 0.f && (rc = scatter_into(h, dg, -lr, h->w, false, st)) != PSS_OK) return rc;
     } else {
@@ -554,7 +693,18 @@ pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, 
     const float* dg = nullptr;
     pss_status rc = device_view(grad_out, (size_t)nbags * (size_t)h->dp.d, h->st_grad, st, &dg);
     if (rc != PSS_OK) return rc;
-    if (h->accum == PSS_ACCUM_F32) {
+    const bool sorted = h->batch_emitted && want_sorted(h);
+    h->last_path = sorted ? PSS_PATH_SORTED : PSS_PATH_ATOMIC;
+    if (sorted) {
+        const int64_t saved = h->accum;
+        h->accum = PSS_ACCUM_F64;
+        rc = ensure_grad(h, st);
+        h->accum = saved;
+        if (rc != PSS_OK) return rc;
+        if ((rc = sorted_into64(h, dg, false, st)) != PSS_OK) return rc;
+        LaunchScope ls(h, PSS_K_MISC, st);
+        PSS_TRY(launch_grad_export(h->g64, grad, h->dp.M, h->sm_count, st));
+    } else if (h->accum == PSS_ACCUM_F32) {
         PSS_TRY(cudaMemsetAsync(grad, 0, sizeof(float) * (size_t)h->dp.M, st));
         if ((rc = scatter_into(h, dg, 1.0f, grad, false, st)) != PSS_OK) return rc;
     } else {
@@ -614,6 +764,7 @@ pss_status pss_get_error(pss_handle* h, int64_t* first_bad_index, pss_stream str
 
 pss_status pss_get_info(pss_handle* h, pss_info* info) {
     if (!h || !info) return PSS_ERR_INVALID_ARG;
+    poll_stats(h);
     info->T = h->dp.T;
     info->d = h->dp.d;
     info->M = h->dp.M;

@@ -41,14 +41,40 @@ struct Touched {
     int64_t cap;
 };
 
+// Buffers of the sorted backward path (see pss_sorted.cu).
+struct SortedBuffers {
+    uint32_t* pair_x;             // nnz*J buckets written by the forward (0xffffffff: bad id)
+    uint32_t* q_row;              // nnz output rows b*T + t written by the forward
+    uint32_t* cnt;                // R per-bucket counts, filled by the forward
+    uint32_t* start;              // R + 1 bucket starts
+    uint32_t* bsum;               // per scan chunk: entries, then their exclusive prefix
+    uint32_t* btask;              // per scan chunk: tasks, then their exclusive prefix
+    uint32_t* bnz;                // per scan chunk: non-empty buckets
+    unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets, [2] tasks
+    uint2* tasks;                 // (bucket, piece) of every reduce task
+    uint32_t* sorted_r;           // nnz*J, row*J + j of each entry in bucket order
+};
+int64_t sorted_scan_blocks(int64_t R);
+int64_t sorted_max_tasks(int64_t R, int64_t npairs);
+cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, cudaStream_t st);
+cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
+                                  cudaStream_t st);
+cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                                 const DevParams& p, double* g, const Touched* touched,
+                                 int sm_count, cudaStream_t st);
+
 // Kernel launchers (return the CUDA launch error).  `grid_cap` bounds the
 // grid of grid-stride kernels; 0 lets the launcher decide.
 cudaError_t launch_locations(const DevParams& p, const int64_t* idx, int64_t nnz,
                              const int64_t* off, int64_t B, int64_t* locs, DevError* err,
                              int sm_count, cudaStream_t st);
+// Forward; when pair_x / q_row / cnt are given it also writes every pair's
+// bucket, every id's output row and the per-bucket counts for the sorted
+// backward path (cnt must be zero on entry).
 cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
-                           DevError* err, int sm_count, cudaStream_t st);
+                           DevError* err, uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt,
+                           int sm_count, cudaStream_t st);
 // Backward scatter into an fp32 target (scale applied to grad_out) or into an
 // fp64 accumulator (scale 1).
 cudaError_t launch_scatter(const DevParams& p, const RowLayout& lay, const int64_t* idx,

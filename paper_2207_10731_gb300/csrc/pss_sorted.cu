@@ -1,0 +1,350 @@
+// Sorted backward path (the sparse branch of Algorithm 1: find the distinct
+// locations, sum the contributions of each, then apply them).
+//
+// Input, written by the forward pass of the same batch:
+//   pair_x[p]  bucket x of pair p = q*J + j (block start G*x), or 0xffffffff
+//              for an id outside its table;
+//   q_row[q]   output row b*T + t of the bag that holds id q;
+//   cnt[x]     number of valid pairs with bucket x (the forward zeroes and
+//              fills it while it hashes).
+// Steps (all on the caller's stream):
+//   1. scan     start[x] = sum of cnt[y] for y < x; every non-empty bucket is
+//               cut into tasks of at most kPiece entries, listed as (x, k);
+//               statistics: valid pairs, distinct buckets, tasks;
+//   2. scatter  each pair takes slot start[x] + (--cnt[x]) of sorted_r, which
+//               holds r = row*J + j (the upstream-gradient chunk to add);
+//   3. reduce   one group of lanes per task: the lanes own 16-byte columns of
+//               the block, add the task's chunks with compensated (Kahan)
+//               fp32 sums, and add the result once into the fp64 gradient
+//               accumulator g[G*x + z] -- one reduction per task and element,
+//               instead of one per contribution, with no hot-address queues.
+// The optimizer pass over g follows (pss_kernels.cu).
+#include <climits>
+
+#include "pss_device.cuh"
+#include "pss_internal.h"
+
+namespace pss {
+namespace {
+
+constexpr uint32_t kBad = 0xffffffffu;
+constexpr int kScanThreads = 1024;
+constexpr int kScanPerThread = 8;
+constexpr int kScanChunk = kScanThreads * kScanPerThread;
+constexpr uint32_t kPiece = 64;   // entries per reduce task
+constexpr int kRU = 4;            // entries in flight per group
+
+__device__ __forceinline__ uint32_t ntasks_of(uint32_t c) { return (c + kPiece - 1) / kPiece; }
+
+// Block-wide exclusive scan of one value per thread (kScanThreads threads).
+__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s_warp,
+                                                         uint32_t* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) s_warp[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+        const uint32_t w = (lane < (kScanThreads >> 5)) ? s_warp[lane] : 0u;
+        uint32_t ws = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xffffffffu, ws, o);
+            if (lane >= o) ws += y;
+        }
+        if (lane < (kScanThreads >> 5)) s_warp[lane] = ws - w;
+        if (lane == 31) s_warp[32] = ws;
+    }
+    __syncthreads();
+    const uint32_t r = s_warp[warp] + x - v;
+    *total = s_warp[32];
+    __syncthreads();
+    return r;
+}
+
+// Per chunk of kScanChunk counters: entries, tasks and non-empty buckets.
+__global__ void __launch_bounds__(kScanThreads)
+k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict__ bsum,
+              uint32_t* __restrict__ btask, uint32_t* __restrict__ bnz) {
+    __shared__ uint32_t s_warp[33];
+    const int64_t base = (int64_t)blockIdx.x * kScanChunk;
+    uint32_t sum = 0, nt = 0, nz = 0;
+#pragma unroll
+    for (int i = 0; i < kScanPerThread; ++i) {
+        const int64_t e = base + (int64_t)i * kScanThreads + threadIdx.x;
+        const uint32_t c = (e < R) ? cnt[e] : 0u;
+        sum += c;
+        nt += ntasks_of(c);
+        nz += (c != 0u);
+    }
+    uint32_t tot;
+    block_exclusive_scan(sum, s_warp, &tot);
+    if (threadIdx.x == 0) bsum[blockIdx.x] = tot;
+    block_exclusive_scan(nt, s_warp, &tot);
+    if (threadIdx.x == 0) btask[blockIdx.x] = tot;
+    block_exclusive_scan(nz, s_warp, &tot);
+    if (threadIdx.x == 0) bnz[blockIdx.x] = tot;
+}
+
+// Exclusive scans of the chunk sums (one block).  stats[0] = valid pairs,
+// stats[1] = distinct buckets, stats[2] = tasks.
+__global__ void __launch_bounds__(kScanThreads)
+k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ btask,
+           const uint32_t* __restrict__ bnz, int64_t nblk, unsigned long long* __restrict__ stats) {
+    __shared__ uint32_t s_warp[33];
+    __shared__ uint32_t s_carry[2];
+    __shared__ unsigned long long s_nz[kScanThreads / 32];
+    if (threadIdx.x < 2) s_carry[threadIdx.x] = 0;
+    __syncthreads();
+    unsigned long long nz = 0;
+    for (int64_t b0 = 0; b0 < nblk; b0 += kScanThreads) {
+        const int64_t b = b0 + threadIdx.x;
+        const bool in = b < nblk;
+        const uint32_t v = in ? bsum[b] : 0u;
+        const uint32_t t = in ? btask[b] : 0u;
+        nz += in ? bnz[b] : 0u;
+        uint32_t tot_v, tot_t;
+        const uint32_t ex_v = block_exclusive_scan(v, s_warp, &tot_v);
+        const uint32_t ex_t = block_exclusive_scan(t, s_warp, &tot_t);
+        const uint32_t cv = s_carry[0], ct = s_carry[1];
+        if (in) {
+            bsum[b] = cv + ex_v;
+            btask[b] = ct + ex_t;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            s_carry[0] = cv + tot_v;
+            s_carry[1] = ct + tot_t;
+        }
+        __syncthreads();
+    }
+    for (int o = 16; o > 0; o >>= 1) nz += __shfl_down_sync(0xffffffffu, nz, o);
+    if ((threadIdx.x & 31) == 0) s_nz[threadIdx.x >> 5] = nz;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned long long total_nz = 0;
+        for (int w = 0; w < (kScanThreads >> 5); ++w) total_nz += s_nz[w];
+        stats[0] = s_carry[0];
+        stats[1] = total_nz;
+        stats[2] = s_carry[1];
+    }
+}
+
+// start[x] (and start[R]); the task list entries (x, k) of every bucket.
+__global__ void __launch_bounds__(kScanThreads)
+k_scan_apply(const uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __restrict__ bsum,
+             const uint32_t* __restrict__ btask, uint32_t* __restrict__ start,
+             uint2* __restrict__ tasks) {
+    __shared__ uint32_t s_warp[33];
+    const int64_t base = (int64_t)blockIdx.x * kScanChunk;
+    uint32_t c[kScanPerThread];
+    uint32_t sum = 0, nt = 0;
+#pragma unroll
+    for (int i = 0; i < kScanPerThread; ++i) {
+        const int64_t e = base + (int64_t)threadIdx.x * kScanPerThread + i;
+        c[i] = (e < R) ? cnt[e] : 0u;
+        sum += c[i];
+        nt += ntasks_of(c[i]);
+    }
+    uint32_t tot;
+    uint32_t run = bsum[blockIdx.x] + block_exclusive_scan(sum, s_warp, &tot);
+    uint32_t trun = btask[blockIdx.x] + block_exclusive_scan(nt, s_warp, &tot);
+#pragma unroll
+    for (int i = 0; i < kScanPerThread; ++i) {
+        const int64_t e = base + (int64_t)threadIdx.x * kScanPerThread + i;
+        if (e < R) {
+            start[e] = run;
+            const uint32_t n = ntasks_of(c[i]);
+            for (uint32_t k = 0; k < n; ++k) tasks[trun + k] = make_uint2((uint32_t)e, k);
+            trun += n;
+        }
+        run += c[i];
+        if (e == R - 1) start[R] = run;
+    }
+}
+
+// Slot of every valid pair; cnt counts back down to zero.
+__global__ void __launch_bounds__(kThreads)
+k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
+               int J, int log2J, const uint32_t* __restrict__ start, uint32_t* __restrict__ cnt,
+               uint32_t* __restrict__ sorted_r) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < npairs; p += stride) {
+        const uint32_t x = __ldg(pair_x + p);
+        if (x == kBad) continue;
+        const uint32_t pp = (uint32_t)p;            // npairs < 2^32 on this path
+        const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
+        const uint32_t j = pp - q * (uint32_t)J;
+        const uint32_t r = __ldg(q_row + q) * (uint32_t)J + j;
+        const uint32_t slot = __ldg(start + x) + atomicSub(cnt + x, 1u) - 1u;
+        sorted_r[slot] = r;
+    }
+}
+
+// Reduce: one group of gs lanes per task; lane lg owns columns lg + k*gs of
+// VW elements of the L-element block.
+template <int VW, int KC, bool JPOW2>
+__global__ void __launch_bounds__(kThreads)
+k_task_reduce(const uint2* __restrict__ tasks, const uint32_t* __restrict__ start,
+              const uint32_t* __restrict__ sorted_r, const unsigned long long* __restrict__ stats,
+              const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
+              double* __restrict__ g, Touched tc, int log2gs) {
+    using V = Vec<VW>;
+    using VT = typename V::T;
+    extern __shared__ __align__(16) float s_stage[];   // [groups per CTA][L]
+    const int64_t ntasks = (int64_t)stats[2];
+    const int lane = threadIdx.x & 31;
+    const int gs = 1 << log2gs;
+    const int lg = lane & (gs - 1);
+    const int gpw = 32 >> log2gs;
+    const int grp = (threadIdx.x >> 5) * gpw + (lane >> log2gs);
+    float* stage = s_stage + grp * L;
+    const unsigned gmask = (gs == 32) ? 0xffffffffu
+                                      : (((1u << gs) - 1u) << ((lane >> log2gs) << log2gs));
+    const int64_t gstride = (int64_t)gridDim.x * kWarps * gpw;
+    for (int64_t t = (int64_t)blockIdx.x * kWarps * gpw + grp; t < ntasks; t += gstride) {
+        const uint2 tk = __ldg(tasks + t);
+        const uint32_t x = tk.x;
+        const uint32_t e0 = __ldg(start + x) + tk.y * kPiece;
+        const uint32_t eb = __ldg(start + x + 1);
+        const uint32_t e1 = (e0 + kPiece < eb) ? e0 + kPiece : eb;
+        float s[KC][VW], c[KC][VW];
+#pragma unroll
+        for (int k = 0; k < KC; ++k)
+#pragma unroll
+            for (int i = 0; i < VW; ++i) s[k][i] = c[k][i] = 0.f;
+        for (uint32_t e = e0; e < e1; e += kRU) {
+            VT v[kRU][KC];
+#pragma unroll
+            for (int u = 0; u < kRU; ++u) {
+#pragma unroll
+                for (int k = 0; k < KC; ++k)
+#pragma unroll
+                    for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
+                if (e + u < e1) {
+                    const uint32_t r = __ldg(sorted_r + e + u);
+                    const uint32_t row = JPOW2 ? (r >> log2J) : r / (uint32_t)J;
+                    const int j = (int)(r - row * (uint32_t)J);
+                    const int Lj = (d - j * Z) < Z ? (d - j * Z) : Z;
+                    const float* src = gout + (int64_t)row * d + j * Z;
+#pragma unroll
+                    for (int k = 0; k < KC; ++k) {
+                        const int col = (lg + k * gs) * VW;
+                        if (col < Lj) v[u][k] = V::ldcs(src + col);
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kRU; ++u)
+#pragma unroll
+                for (int k = 0; k < KC; ++k)
+#pragma unroll
+                    for (int i = 0; i < VW; ++i) kahan_add(s[k][i], c[k][i], V::get(v[u][k], i));
+        }
+        // transpose through shared memory so that each fp64 reduction
+        // instruction covers consecutive elements
+#pragma unroll
+        for (int k = 0; k < KC; ++k) {
+            const int col = (lg + k * gs) * VW;
+#pragma unroll
+            for (int i = 0; i < VW; ++i)
+                if (col + i < L) stage[col + i] = s[k][i];
+        }
+        __syncwarp(gmask);
+        double* base = g + (int64_t)x * G;
+        for (int z = lg; z < L; z += gs) {
+            const float val = stage[z];
+            if (val != 0.f) red_add_f64(base + z, (double)val);
+        }
+        if (tc.bitmap && lg == 0) mark_touched(tc, x);
+        __syncwarp(gmask);
+    }
+}
+
+template <int VW, int KC>
+cudaError_t reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                        const DevParams& p, double* g, const Touched& tc, int log2gs,
+                        int sm_count, cudaStream_t st) {
+    const int log2J = (p.J & (p.J - 1)) == 0 ? ceil_log2(p.J) : -1;
+    const int gpc = kWarps * (32 >> log2gs);
+    const size_t smem = sizeof(float) * (size_t)gpc * (size_t)p.L;
+    // tasks <= valid pairs <= npairs; the exact count is read on the device
+    const int64_t work_blocks = (npairs + gpc - 1) / gpc;
+    if (log2J >= 0) {
+        const int grid = grid_for(k_task_reduce<VW, KC, true>, sm_count, work_blocks, smem);
+        k_task_reduce<VW, KC, true><<<grid, kThreads, smem, st>>>(
+            sb.tasks, sb.start, sb.sorted_r, sb.stats, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, tc,
+            log2gs);
+    } else {
+        const int grid = grid_for(k_task_reduce<VW, KC, false>, sm_count, work_blocks, smem);
+        k_task_reduce<VW, KC, false><<<grid, kThreads, smem, st>>>(
+            sb.tasks, sb.start, sb.sorted_r, sb.stats, gout, p.d, p.Z, p.J, 0, p.L, p.G, g, tc,
+            log2gs);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int64_t sorted_scan_blocks(int64_t R) { return (R + kScanChunk - 1) / kScanChunk; }
+
+int64_t sorted_max_tasks(int64_t R, int64_t npairs) {
+    return (R < npairs ? R : npairs) + npairs / kPiece + 1;
+}
+
+cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, cudaStream_t st) {
+    const int64_t nblk = sorted_scan_blocks(R);
+    k_scan_reduce<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.btask, sb.bnz);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_scan_top<<<1, kScanThreads, 0, st>>>(sb.bsum, sb.btask, sb.bnz, nblk, sb.stats);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_scan_apply<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.btask, sb.start,
+                                                          sb.tasks);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
+                                  cudaStream_t st) {
+    const int log2J = (J & (J - 1)) == 0 ? ceil_log2(J) : -1;
+    const int grid = grid_for(k_sort_scatter, sm_count, (npairs + kThreads - 1) / kThreads);
+    k_sort_scatter<<<grid, kThreads, 0, st>>>(sb.pair_x, npairs, sb.q_row, J, log2J, sb.start,
+                                              sb.cnt, sb.sorted_r);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                                 const DevParams& p, double* g, const Touched* touched,
+                                 int sm_count, cudaStream_t st) {
+    const Touched tc = touched ? *touched : Touched{};
+    const bool vec = (p.Z % 4 == 0) && (p.d % 4 == 0) && (((uintptr_t)gout & 15u) == 0);
+    const int vw = vec ? 4 : 1;
+    const int V = (p.L + vw - 1) / vw;
+    const int log2gs = V <= 32 ? ceil_log2(V) : 5;
+    const int kc = V <= 32 ? 1 : (1 << ceil_log2((V + 31) / 32));
+#define PSS_RD(VW, KC) return reduce_inst<VW, KC>(sb, npairs, gout, p, g, tc, log2gs, sm_count, st)
+    if (vec) {
+        switch (kc) {
+            case 1: PSS_RD(4, 1);
+            case 2: PSS_RD(4, 2);
+            case 4: PSS_RD(4, 4);
+        }
+    } else {
+        switch (kc) {
+            case 1: PSS_RD(1, 1);
+            case 2: PSS_RD(1, 2);
+            case 4: PSS_RD(1, 4);
+            case 8: PSS_RD(1, 8);
+            case 16: PSS_RD(1, 16);
+        }
+    }
+#undef PSS_RD
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace pss

@@ -45,27 +45,34 @@ struct TileGeom {
 
 // Stage the offsets of tile (t, b0) into s_off; returns false (and zeroes the
 // tile's rows when `out` is given) if the offsets are malformed.
+// s_flags bit 0: malformed offsets; bit 1: some bag holds more than one id.
 __device__ __forceinline__ bool stage_offsets(const int64_t* __restrict__ off, int64_t s0, int nb,
-                                              int64_t nnz, int64_t* s_off, int* s_bad,
-                                              DevError* err) {
-    if (threadIdx.x == 0) *s_bad = 0;
+                                              int64_t nnz, int64_t* s_off, int* s_flags,
+                                              DevError* err, bool* one_hot = nullptr) {
+    if (threadIdx.x == 0) *s_flags = 0;
     for (int i = threadIdx.x; i <= nb; i += kThreads) s_off[i] = __ldg(off + s0 + i);
     __syncthreads();
+    int f = 0;
     for (int i = threadIdx.x; i < nb; i += kThreads) {
         const int64_t a = s_off[i], c = s_off[i + 1];
-        if (a < 0 || c < a || c > nnz) *s_bad = 1;
+        if (a < 0 || c < a || c > nnz) f |= 1;
+        if (c - a > 1) f |= 2;
     }
+    if (f) atomicOr(s_flags, f);
     __syncthreads();
-    const bool bad = *s_bad != 0;
-    if (bad && threadIdx.x == 0) record_bad_offsets(err);
-    return !bad;
+    const int flags = *s_flags;
+    if ((flags & 1) && threadIdx.x == 0) record_bad_offsets(err);
+    if (one_hot) *one_hot = (flags & 2) == 0;
+    return !(flags & 1);
 }
 
 // Hash every (id, chunk) pair of ids [qc0, qc0 + nq) of table t into s_x.
 template <typename XT, bool TOUCH>
 __device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t* __restrict__ idx,
                                               int t, uint64_t card, int64_t qc0, int nq, XT* s_x,
-                                              DevError* err, const Touched& tc) {
+                                              DevError* err, const Touched& tc,
+                                              uint32_t* __restrict__ pair_x = nullptr,
+                                              uint32_t* __restrict__ cnt = nullptr) {
     const int npairs = nq * p.J;
     for (int k = threadIdx.x; k < npairs; k += kThreads) {
         const int qi = k / p.J;
@@ -80,8 +87,10 @@ __device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t*
             const uint64_t b = hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
             x = (XT)b;
             if (TOUCH) mark_touched(tc, b);
+            if (cnt) atomicAdd(cnt + b, 1u);
         }
         s_x[k] = x;
+        if (pair_x) pair_x[qc0 * p.J + k] = (uint32_t)x;
     }
 }
 
@@ -90,7 +99,9 @@ template <int VW, int KC, typename XT>
 __global__ void __launch_bounds__(kThreads)
 k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                 const int64_t* __restrict__ off, int64_t B, const float* __restrict__ w,
-                float* __restrict__ out, DevError* err, int log2gs, TileGeom tg) {
+                float* __restrict__ out, DevError* err, uint32_t* __restrict__ pair_x,
+                uint32_t* __restrict__ q_row, uint32_t* __restrict__ cnt, int log2gs,
+                TileGeom tg) {
     using V = Vec<VW>;
     using VT = typename V::T;
     extern __shared__ __align__(16) unsigned char smem[];
@@ -118,7 +129,8 @@ k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
         float* obase = out + ((b0 * p.T) + t) * (int64_t)p.d;   // row of bag b0
         const int64_t ostride = (int64_t)p.T * p.d;               // next bag row
 
-        if (!stage_offsets(off, s0, nb, nnz, s_off, &s_bad, err)) {
+        bool one_hot = false;
+        if (!stage_offsets(off, s0, nb, nnz, s_off, &s_bad, err, &one_hot)) {
             for (int bi = gb0; bi < gb1; ++bi)
 #pragma unroll
                 for (int k = 0; k < KC; ++k) {
@@ -133,6 +145,42 @@ k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
         }
         const uint64_t card = (uint64_t)__ldg(p.cards + t);
         const int64_t qa = s_off[0], qb = s_off[nb];
+        if (one_hot && qb - qa <= tg.qc) {
+            // every bag holds at most one id: no accumulation, one load per bag
+            stage_buckets<XT, false>(p, idx, t, card, qa, (int)(qb - qa), s_x, err, none, pair_x,
+                                     cnt);
+            __syncthreads();
+            for (int b = gb0; b < gb1; b += kU) {
+                VT v[kU][KC];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int bb = b + u;
+                    int64_t q = -1;
+                    if (bb < gb1 && s_off[bb + 1] > s_off[bb]) q = s_off[bb];
+#pragma unroll
+                    for (int k = 0; k < KC; ++k) {
+#pragma unroll
+                        for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
+                        if (q >= 0 && col.v[k]) {
+                            const XT x = s_x[(int)(q - qa) * J + col.j[k]];
+                            if (x != Invalid<XT>::v) v[u][k] = V::ldg(w + G * (uint64_t)x + col.z[k]);
+                        }
+                    }
+                    if (q >= 0 && q_row && lg == 0) q_row[q] = (uint32_t)((b0 + bb) * p.T + t);
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int bb = b + u;
+                    if (bb >= gb1) break;
+                    float* orow = obase + bb * ostride;
+#pragma unroll
+                    for (int k = 0; k < KC; ++k)
+                        if (col.v[k]) V::stcs(orow + col.e[k], v[u][k]);
+                }
+            }
+            __syncthreads();
+            continue;
+        }
         const int64_t gq0 = s_off[gb0], gq1 = s_off[gb1];
         int bi = gb0;
         int64_t qend = (gb0 < gb1) ? s_off[gb0 + 1] : 0;
@@ -159,7 +207,7 @@ k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
 
         for (int64_t qc0 = qa; qc0 < qb; qc0 += tg.qc) {
             const int nq = (int)((qb - qc0) < tg.qc ? (qb - qc0) : tg.qc);
-            stage_buckets<XT, false>(p, idx, t, card, qc0, nq, s_x, err, none);
+            stage_buckets<XT, false>(p, idx, t, card, qc0, nq, s_x, err, none, pair_x, cnt);
             __syncthreads();
             const int64_t qlo = gq0 > qc0 ? gq0 : qc0;
             const int64_t qhi = gq1 < qc0 + nq ? gq1 : qc0 + nq;
@@ -185,6 +233,7 @@ k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                         ++bi;
                         qend = s_off[bi + 1];
                     }
+                    if (q_row && lg == 0) q_row[q + u] = (uint32_t)((b0 + bi) * p.T + t);
 #pragma unroll
                     for (int k = 0; k < KC; ++k)
 #pragma unroll
@@ -321,13 +370,14 @@ size_t tile_smem(const TileGeom& g, const DevParams& p, size_t xbytes) {
 template <int VW, int KC, typename XT>
 cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                      const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
-                     int sm_count, cudaStream_t st) {
+                     uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt, int sm_count,
+                     cudaStream_t st) {
     const TileGeom tg = tile_geom(p, lay, B, sizeof(XT));
     const size_t smem = tile_smem(tg, p, sizeof(XT));
     const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
     const int grid = grid_for(k_forward_tiled<VW, KC, XT>, sm_count, ntiles, smem);
     k_forward_tiled<VW, KC, XT><<<grid, kThreads, smem, st>>>(p, idx, nnz, off, B, w, out, err,
-                                                              lay.log2gs, tg);
+                                                              pair_x, q_row, cnt, lay.log2gs, tg);
     return cudaGetLastError();
 }
 
@@ -347,10 +397,13 @@ cudaError_t sc_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx
 template <int VW, int KC>
 cudaError_t fwd_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                   const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
-                  int sm_count, cudaStream_t st) {
+                  uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt, int sm_count,
+                  cudaStream_t st) {
     if (p.R < 0xffffffffull)
-        return fwd_inst<VW, KC, uint32_t>(p, lay, idx, nnz, off, B, w, out, err, sm_count, st);
-    return fwd_inst<VW, KC, uint64_t>(p, lay, idx, nnz, off, B, w, out, err, sm_count, st);
+        return fwd_inst<VW, KC, uint32_t>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row,
+                                          cnt, sm_count, st);
+    return fwd_inst<VW, KC, uint64_t>(p, lay, idx, nnz, off, B, w, out, err, nullptr, nullptr,
+                                      nullptr, sm_count, st);
 }
 
 template <int VW, int KC, typename AT>
@@ -377,8 +430,10 @@ cudaError_t sc_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, i
 
 cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
-                           DevError* err, int sm_count, cudaStream_t st) {
-#define PSS_FW(VW, KC) return fwd_x<VW, KC>(p, lay, idx, nnz, off, B, w, out, err, sm_count, st)
+                           DevError* err, uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt,
+                           int sm_count, cudaStream_t st) {
+#define PSS_FW(VW, KC) \
+    return fwd_x<VW, KC>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row, cnt, sm_count, st)
     if (lay.vw == 4) {
         switch (lay.kc) {
             case 1: PSS_FW(4, 1);

@@ -115,10 +115,15 @@ def test_forward_dyadic_bit_exact(name, B):
 
 # --------------------------------------------------------------------------
 # gradient (row a4): lr = 0 capture through pss_backward_grad
+PATHS = {"auto": binding.PATH_AUTO, "atomic": binding.PATH_ATOMIC, "sorted": binding.PATH_SORTED}
+
+
+@pytest.mark.parametrize("path", list(PATHS))
 @pytest.mark.parametrize("case", FWD_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
-def test_grad_parity(case):
+def test_grad_parity(case, path):
     w = _wl(case)
     h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
     h.forward(*_batch_cuda(w), w.B)
     g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
     ref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
@@ -129,6 +134,8 @@ def test_grad_parity(case):
     rows = w.grad_out.reshape(w.B, w.T, w.d).astype(np.float64).sum(axis=2)
     mass = float((lengths.T * rows).sum())
     assert abs(g.astype(np.float64).sum() - mass) <= 1e-5 * A.sum() + 1e-6
+    if path != "auto":
+        assert h.info()["last_path"] == PATHS[path]
     h.close()
 
 
@@ -169,8 +176,9 @@ def _run_step(w, h, o, wcur, Gcur, batch):
     return gu.host(wg), (gu.host(Gg) if Gg is not None else None), w2, G2, g32, A
 
 
+@pytest.mark.parametrize("path", list(PATHS))
 @pytest.mark.parametrize("case", STEP_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
-def test_step_parity_three_steps(case):
+def test_step_parity_three_steps(case, path):
     case = dict(case)
     opt = case.pop("opt", None)
     lr = case.pop("lr", None)
@@ -180,6 +188,7 @@ def test_step_parity_three_steps(case):
     if lr:
         w.lr = lr
     h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
     wcur = w.w0.copy()
     Gcur = np.zeros(w.M, dtype=np.float32)
     cfg = wl.CONFIGS[case["name"]]
@@ -200,11 +209,13 @@ def test_step_parity_three_steps(case):
     h.close()
 
 
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
 @pytest.mark.parametrize("opt", ["sgd", "adagrad"])
-def test_step_dyadic_bit_exact(opt):
+def test_step_dyadic_bit_exact(opt, path):
     w = wl.make_workload("kaggle", B=1024, grad="dyadic", w0="dyadic")
     w.lr = 0.125
     h, o = gu.make_pair(w, opt=opt)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
     h.forward(*_batch_cuda(w), w.B)
     h.backward_update(gu.cuda(w.grad_out), w.lr)
     wg, Gg = h.get_state()
@@ -216,21 +227,44 @@ def test_step_dyadic_bit_exact(opt):
     h.close()
 
 
-def test_dense_and_touched_updates_identical():
-    # Same exact gradient (dyadic inputs), two ways of visiting M: same bits.
+def test_dense_and_touched_updates_identical_on_both_paths():
+    # Same exact gradient (dyadic inputs), two ways of visiting M and two
+    # backward paths: same bits.
     w = wl.make_workload("tb", B=2048, grad="dyadic", w0="dyadic")
     res = []
-    for mode in (binding.UPDATE_DENSE, binding.UPDATE_TOUCHED):
+    for mode, path in [(binding.UPDATE_DENSE, binding.PATH_ATOMIC),
+                       (binding.UPDATE_TOUCHED, binding.PATH_ATOMIC),
+                       (binding.UPDATE_DENSE, binding.PATH_SORTED),
+                       (binding.UPDATE_TOUCHED, binding.PATH_SORTED)]:
         h, _ = gu.make_pair(w, opt="adagrad")
         h.set_option(binding.OPT_UPDATE_MODE, mode)
+        h.set_option(binding.OPT_BACKWARD_PATH, path)
         for _ in range(2):
             h.forward(*_batch_cuda(w), w.B)
             h.backward_update(gu.cuda(w.grad_out), 0.01)
         wg, Gg = h.get_state()
         res.append((gu.host(wg), gu.host(Gg)))
         h.close()
-    np.testing.assert_array_equal(res[0][0], res[1][0])
-    np.testing.assert_array_equal(res[0][1], res[1][1])
+    for r in res[1:]:
+        np.testing.assert_array_equal(res[0][0], r[0])
+        np.testing.assert_array_equal(res[0][1], r[1])
+
+
+def test_sorted_path_reports_collision_rate():
+    # rho = 1 - distinct blocks / (ids * chunks), from the sorted pass's counters
+    t = gu.torch()
+    w = wl.make_workload("tb", B=4096)
+    h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    h.forward(*_batch_cuda(w), w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    t.cuda.synchronize()
+    info = h.info()
+    locs, _ = o.locations(w.indices, w.offsets, w.B)
+    want = 1.0 - np.unique(locs).shape[0] / locs.shape[0]
+    assert info["last_path"] == binding.PATH_SORTED
+    assert abs(info["last_collision_rate"] - want) < 1e-12
+    h.close()
 
 
 @pytest.mark.parametrize("name,B", [("microbench", 10240), ("multihot", 4096), ("tb", 8192)])
@@ -396,12 +430,14 @@ def test_host_buffers_match_device_buffers():
 
 # --------------------------------------------------------------------------
 # errors: reported, never a trap
-def test_out_of_range_ids_are_skipped_and_reported():
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
+def test_out_of_range_ids_are_skipped_and_reported(path):
     w = wl.make_workload("tiny")
     idx = w.indices.copy()
     idx[100] = 5000          # beyond the 1000-id table
     idx[37] = -3
     h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
     out = gu.host(h.forward(gu.cuda(idx), gu.cuda(w.offsets), w.B)).ravel()
     st, first = h.get_error()
     assert st == binding.PSS_ERR_INDEX_RANGE and first == 37
@@ -409,6 +445,11 @@ def test_out_of_range_ids_are_skipped_and_reported():
     assert bad == 37
     np.testing.assert_array_equal(out, ref)
     assert h.get_error() == (binding.PSS_OK, -1)     # cleared by the read
+    # the backward skips the same ids
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    gref = o.grad(idx, w.offsets, w.B, w.grad_out)
+    A = o.grad(idx, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g, gref, A)
     h.close()
 
 
@@ -460,6 +501,7 @@ def test_profile_and_launch_counts():
     w = wl.make_workload("kaggle")
     h, _ = gu.make_pair(w)
     h.set_option(binding.OPT_PROFILE, 1)
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_ATOMIC)
     idx, off = _batch_cuda(w)
     go = gu.cuda(w.grad_out)
     before = h.info()["kernel_launches"]
@@ -470,4 +512,12 @@ def test_profile_and_launch_counts():
     n_s, ms_s = h.profile(binding.K_SCATTER)
     assert n_f == 3 and n_s == 3 and ms_f > 0 and ms_s > 0
     assert h.info()["kernel_launches"] - before == 9     # forward, scatter, update
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    h.reset_profile()
+    before = h.info()["kernel_launches"]
+    h.forward(idx, off, w.B)
+    h.backward_update(go, w.lr)
+    assert h.profile(binding.K_SORT)[0] == 1 and h.profile(binding.K_REDUCE)[0] == 1
+    # forward (which also counts buckets), 3 scan kernels, scatter, reduce, update
+    assert h.info()["kernel_launches"] - before == 7
     h.close()
