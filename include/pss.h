@@ -100,6 +100,8 @@ typedef enum {
     PSS_OPT_ACCUM = 5
 } pss_option;
 
+
+
 enum { PSS_ACCUM_F64 = 0, PSS_ACCUM_F32 = 1 };
 
 enum { PSS_PATH_AUTO = 0, PSS_PATH_ATOMIC = 1, PSS_PATH_SORTED = 2 };

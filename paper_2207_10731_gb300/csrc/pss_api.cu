@@ -257,28 +257,23 @@ pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {
         PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)R, st));
         PSS_TRY(cudaMalloc(&h->sb.start, sizeof(uint32_t) * (size_t)(R + 1)));
         PSS_TRY(cudaMalloc(&h->sb.bsum, sizeof(uint32_t) * (size_t)nblk));
-        PSS_TRY(cudaMalloc(&h->sb.btask, sizeof(uint32_t) * (size_t)nblk));
         PSS_TRY(cudaMalloc(&h->sb.bnz, sizeof(uint32_t) * (size_t)nblk));
-        PSS_TRY(cudaMalloc(&h->sb.stats, 3 * sizeof(unsigned long long)));
-        PSS_TRY(cudaMemsetAsync(h->sb.stats, 0, 3 * sizeof(unsigned long long), st));
+        PSS_TRY(cudaMalloc(&h->sb.stats, 2 * sizeof(unsigned long long)));
+        PSS_TRY(cudaMemsetAsync(h->sb.stats, 0, 2 * sizeof(unsigned long long), st));
         PSS_TRY(cudaMallocHost(&h->stats_host, 2 * sizeof(unsigned long long)));
         h->stats_host[0] = h->stats_host[1] = 0;
         PSS_TRY(cudaEventCreateWithFlags(&h->stats_ev, cudaEventDisableTiming));
         h->sb_counters = true;
     }
     if (h->sb_pairs_cap < npairs) {
-        for (uint32_t** b : {&h->sb.pair_x, &h->sb.sorted_r}) {
-            if (*b) PSS_TRY(cudaFreeAsync(*b, st));
-            *b = nullptr;
-        }
-        if (h->sb.tasks) PSS_TRY(cudaFreeAsync(h->sb.tasks, st));
-        h->sb.tasks = nullptr;
+        if (h->sb.pair_x) PSS_TRY(cudaFreeAsync(h->sb.pair_x, st));
+        if (h->sb.sorted_e) PSS_TRY(cudaFreeAsync(h->sb.sorted_e, st));
+        h->sb.pair_x = nullptr;
+        h->sb.sorted_e = nullptr;
         h->sb_pairs_cap = 0;
-        const size_t bytes = sizeof(uint32_t) * (size_t)(npairs > 0 ? npairs : 1);
-        PSS_TRY(cudaMallocAsync(&h->sb.pair_x, bytes, st));
-        PSS_TRY(cudaMallocAsync(&h->sb.sorted_r, bytes, st));
-        PSS_TRY(cudaMallocAsync(&h->sb.tasks,
-                                sizeof(uint2) * (size_t)sorted_max_tasks(R, npairs), st));
+        const size_t n = (size_t)(npairs > 0 ? npairs : 1);
+        PSS_TRY(cudaMallocAsync(&h->sb.pair_x, sizeof(uint32_t) * n, st));
+        PSS_TRY(cudaMallocAsync(&h->sb.sorted_e, sizeof(unsigned long long) * n, st));
         h->sb_pairs_cap = npairs;
     }
     if (h->sb_ids_cap < nnz) {
@@ -433,8 +428,8 @@ pss_status pss_destroy(pss_handle* h) {
     cudaFree(h->touched.list);
     cudaFree(h->touched.count);
     for (void* b : {(void*)h->sb.pair_x, (void*)h->sb.q_row, (void*)h->sb.cnt, (void*)h->sb.start,
-                    (void*)h->sb.bsum, (void*)h->sb.btask, (void*)h->sb.bnz, (void*)h->sb.stats,
-                    (void*)h->sb.tasks, (void*)h->sb.sorted_r})
+                    (void*)h->sb.bsum, (void*)h->sb.bnz, (void*)h->sb.stats,
+                    (void*)h->sb.sorted_e})
         if (b) cudaFree(b);
     if (h->stats_host) cudaFreeHost(h->stats_host);
     if (h->stats_ev) cudaEventDestroy(h->stats_ev);

@@ -48,14 +48,11 @@ struct SortedBuffers {
     uint32_t* cnt;                // R per-bucket counts, filled by the forward
     uint32_t* start;              // R + 1 bucket starts
     uint32_t* bsum;               // per scan chunk: entries, then their exclusive prefix
-    uint32_t* btask;              // per scan chunk: tasks, then their exclusive prefix
     uint32_t* bnz;                // per scan chunk: non-empty buckets
-    unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets, [2] tasks
-    uint2* tasks;                 // (bucket, piece) of every reduce task
-    uint32_t* sorted_r;           // nnz*J, row*J + j of each entry in bucket order
+    unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets
+    unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j) in bucket order
 };
 int64_t sorted_scan_blocks(int64_t R);
-int64_t sorted_max_tasks(int64_t R, int64_t npairs);
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, cudaStream_t st);
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
                                   cudaStream_t st);

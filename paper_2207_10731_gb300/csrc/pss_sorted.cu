@@ -8,16 +8,18 @@
 //   cnt[x]     number of valid pairs with bucket x (the forward zeroes and
 //              fills it while it hashes).
 // Steps (all on the caller's stream):
-//   1. scan     start[x] = sum of cnt[y] for y < x; every non-empty bucket is
-//               cut into tasks of at most kPiece entries, listed as (x, k);
-//               statistics: valid pairs, distinct buckets, tasks;
-//   2. scatter  each pair takes slot start[x] + (--cnt[x]) of sorted_r, which
-//               holds r = row*J + j (the upstream-gradient chunk to add);
-//   3. reduce   one group of lanes per task: the lanes own 16-byte columns of
-//               the block, add the task's chunks with compensated (Kahan)
-//               fp32 sums, and add the result once into the fp64 gradient
-//               accumulator g[G*x + z] -- one reduction per task and element,
-//               instead of one per contribution, with no hot-address queues.
+//   1. scan     start[x] = sum of cnt[y] for y < x (three kernels);
+//               statistics: valid pairs and distinct buckets;
+//   2. scatter  each pair takes slot start[x] + (--cnt[x]) of sorted_e, which
+//               holds (x, r = row*J + j): the bucket and the upstream-gradient
+//               chunk to add;
+//   3. reduce   the sorted entries are cut into tasks of kPiece consecutive
+//               entries; one group of lanes per task owns 16-byte columns of
+//               the block, adds the chunks of each run of equal x with
+//               compensated (Kahan) fp32 sums, and adds every run's sum once
+//               into the fp64 gradient accumulator g[G*x + z] -- one reduction
+//               per run and element instead of one per contribution, and no
+//               queue of reductions on a hot address.
 // The optimizer pass over g follows (pss_kernels.cu).
 #include <climits>
 
@@ -31,10 +33,7 @@ constexpr uint32_t kBad = 0xffffffffu;
 constexpr int kScanThreads = 1024;
 constexpr int kScanPerThread = 8;
 constexpr int kScanChunk = kScanThreads * kScanPerThread;
-constexpr uint32_t kPiece = 64;   // entries per reduce task
 constexpr int kRU = 4;            // entries in flight per group
-
-__device__ __forceinline__ uint32_t ntasks_of(uint32_t c) { return (c + kPiece - 1) / kPiece; }
 
 // Block-wide exclusive scan of one value per thread (kScanThreads threads).
 __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s_warp,
@@ -66,60 +65,49 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s
     return r;
 }
 
-// Per chunk of kScanChunk counters: entries, tasks and non-empty buckets.
+// Per chunk of kScanChunk counters: entries and non-empty buckets.
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict__ bsum,
-              uint32_t* __restrict__ btask, uint32_t* __restrict__ bnz) {
+              uint32_t* __restrict__ bnz) {
     __shared__ uint32_t s_warp[33];
     const int64_t base = (int64_t)blockIdx.x * kScanChunk;
-    uint32_t sum = 0, nt = 0, nz = 0;
+    uint32_t sum = 0, nz = 0;
 #pragma unroll
     for (int i = 0; i < kScanPerThread; ++i) {
         const int64_t e = base + (int64_t)i * kScanThreads + threadIdx.x;
         const uint32_t c = (e < R) ? cnt[e] : 0u;
         sum += c;
-        nt += ntasks_of(c);
         nz += (c != 0u);
     }
     uint32_t tot;
     block_exclusive_scan(sum, s_warp, &tot);
     if (threadIdx.x == 0) bsum[blockIdx.x] = tot;
-    block_exclusive_scan(nt, s_warp, &tot);
-    if (threadIdx.x == 0) btask[blockIdx.x] = tot;
     block_exclusive_scan(nz, s_warp, &tot);
     if (threadIdx.x == 0) bnz[blockIdx.x] = tot;
 }
 
-// Exclusive scans of the chunk sums (one block).  stats[0] = valid pairs,
-// stats[1] = distinct buckets, stats[2] = tasks.
+// Exclusive scan of the chunk sums (one block).  stats[0] = valid pairs,
+// stats[1] = distinct buckets.
 __global__ void __launch_bounds__(kScanThreads)
-k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ btask,
-           const uint32_t* __restrict__ bnz, int64_t nblk, unsigned long long* __restrict__ stats) {
+k_scan_top(uint32_t* __restrict__ bsum, const uint32_t* __restrict__ bnz, int64_t nblk,
+           unsigned long long* __restrict__ stats) {
     __shared__ uint32_t s_warp[33];
-    __shared__ uint32_t s_carry[2];
+    __shared__ uint32_t s_carry;
     __shared__ unsigned long long s_nz[kScanThreads / 32];
-    if (threadIdx.x < 2) s_carry[threadIdx.x] = 0;
+    if (threadIdx.x == 0) s_carry = 0;
     __syncthreads();
     unsigned long long nz = 0;
     for (int64_t b0 = 0; b0 < nblk; b0 += kScanThreads) {
         const int64_t b = b0 + threadIdx.x;
         const bool in = b < nblk;
         const uint32_t v = in ? bsum[b] : 0u;
-        const uint32_t t = in ? btask[b] : 0u;
         nz += in ? bnz[b] : 0u;
-        uint32_t tot_v, tot_t;
+        uint32_t tot_v;
         const uint32_t ex_v = block_exclusive_scan(v, s_warp, &tot_v);
-        const uint32_t ex_t = block_exclusive_scan(t, s_warp, &tot_t);
-        const uint32_t cv = s_carry[0], ct = s_carry[1];
-        if (in) {
-            bsum[b] = cv + ex_v;
-            btask[b] = ct + ex_t;
-        }
+        const uint32_t cv = s_carry;
+        if (in) bsum[b] = cv + ex_v;
         __syncthreads();
-        if (threadIdx.x == 0) {
-            s_carry[0] = cv + tot_v;
-            s_carry[1] = ct + tot_t;
-        }
+        if (threadIdx.x == 0) s_carry = cv + tot_v;
         __syncthreads();
     }
     for (int o = 16; o > 0; o >>= 1) nz += __shfl_down_sync(0xffffffffu, nz, o);
@@ -128,75 +116,100 @@ k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ btask,
     if (threadIdx.x == 0) {
         unsigned long long total_nz = 0;
         for (int w = 0; w < (kScanThreads >> 5); ++w) total_nz += s_nz[w];
-        stats[0] = s_carry[0];
+        stats[0] = s_carry;
         stats[1] = total_nz;
-        stats[2] = s_carry[1];
     }
 }
 
-// start[x] (and start[R]); the task list entries (x, k) of every bucket.
+// start[x] = exclusive prefix of cnt; start[R] = total.
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_apply(const uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __restrict__ bsum,
-             const uint32_t* __restrict__ btask, uint32_t* __restrict__ start,
-             uint2* __restrict__ tasks) {
+             uint32_t* __restrict__ start) {
     __shared__ uint32_t s_warp[33];
     const int64_t base = (int64_t)blockIdx.x * kScanChunk;
     uint32_t c[kScanPerThread];
-    uint32_t sum = 0, nt = 0;
+    uint32_t sum = 0;
 #pragma unroll
     for (int i = 0; i < kScanPerThread; ++i) {
         const int64_t e = base + (int64_t)threadIdx.x * kScanPerThread + i;
         c[i] = (e < R) ? cnt[e] : 0u;
         sum += c[i];
-        nt += ntasks_of(c[i]);
     }
     uint32_t tot;
     uint32_t run = bsum[blockIdx.x] + block_exclusive_scan(sum, s_warp, &tot);
-    uint32_t trun = btask[blockIdx.x] + block_exclusive_scan(nt, s_warp, &tot);
 #pragma unroll
     for (int i = 0; i < kScanPerThread; ++i) {
         const int64_t e = base + (int64_t)threadIdx.x * kScanPerThread + i;
-        if (e < R) {
-            start[e] = run;
-            const uint32_t n = ntasks_of(c[i]);
-            for (uint32_t k = 0; k < n; ++k) tasks[trun + k] = make_uint2((uint32_t)e, k);
-            trun += n;
-        }
+        if (e < R) start[e] = run;
         run += c[i];
         if (e == R - 1) start[R] = run;
     }
 }
 
-// Slot of every valid pair; cnt counts back down to zero.
+// Slot of every valid pair; cnt counts back down to zero.  Lanes of a warp
+// with the same bucket share one atomic (the leader takes n slots at once).
 __global__ void __launch_bounds__(kThreads)
 k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
                int J, int log2J, const uint32_t* __restrict__ start, uint32_t* __restrict__ cnt,
-               uint32_t* __restrict__ sorted_r) {
+               unsigned long long* __restrict__ sorted_e) {
+    const int lane = threadIdx.x & 31;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < npairs; p += stride) {
-        const uint32_t x = __ldg(pair_x + p);
-        if (x == kBad) continue;
+    for (int64_t p0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); p0 < npairs;
+         p0 += stride) {
+        const int64_t p = p0 + lane;
+        const uint32_t x = (p < npairs) ? __ldg(pair_x + p) : kBad;
+        // loads that do not depend on the slot go first, so they overlap the atomic
         const uint32_t pp = (uint32_t)p;            // npairs < 2^32 on this path
         const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
         const uint32_t j = pp - q * (uint32_t)J;
-        const uint32_t r = __ldg(q_row + q) * (uint32_t)J + j;
-        const uint32_t slot = __ldg(start + x) + atomicSub(cnt + x, 1u) - 1u;
-        sorted_r[slot] = r;
+        uint32_t row = 0, st0 = 0;
+        if (x != kBad) {
+            row = __ldg(q_row + q);
+            st0 = __ldg(start + x);
+        }
+        const unsigned peers = __match_any_sync(0xffffffffu, x);
+        const int leader = __ffs(peers) - 1;
+        const int rank = __popc(peers & ((1u << lane) - 1u));
+        uint32_t old = 0;
+        if (x != kBad && lane == leader) old = atomicSub(cnt + x, (uint32_t)__popc(peers));
+        old = __shfl_sync(0xffffffffu, old, leader);
+        if (x == kBad) continue;
+        const uint32_t slot = st0 + old - 1u - (uint32_t)rank;
+        sorted_e[slot] = ((unsigned long long)x << 32) | (row * (uint32_t)J + j);
     }
 }
 
-// Reduce: one group of gs lanes per task; lane lg owns columns lg + k*gs of
-// VW elements of the L-element block.
+// Exact fp32 -> fp64 widening from the IEEE-754 fields (integer pipe): the
+// exponent is re-biased (127 -> 1023) and the 23-bit fraction moved to the top
+// of the 52-bit one.  Zeros, subnormals, infinities and NaNs take the
+// hardware conversion.
+__device__ __forceinline__ double widen(float f) {
+    const uint32_t u = __float_as_uint(f);
+    const uint32_t e = (u >> 23) & 0xffu;
+    if (e == 0u || e == 0xffu) return (double)f;
+    const uint64_t bits = ((uint64_t)(u & 0x80000000u) << 32) |
+                          ((uint64_t)(e + 896u) << 52) | ((uint64_t)(u & 0x7fffffu) << 29);
+    return __longlong_as_double((long long)bits);
+}
+
+// Reduce: one group of gs lanes per task of kPiece sorted entries; lane lg
+// owns columns lg + k*gs of VW elements of the L-element block.  Each run of
+// equal x is summed with compensation (Kahan) and added once into the fp64
+// accumulator through a shared-memory transpose (so that every fp64
+// reduction instruction covers consecutive elements).
+constexpr int64_t kPiece = 64;    // sorted entries per reduce task
+
 template <int VW, int KC, bool JPOW2>
-__global__ void __launch_bounds__(kThreads)
-k_task_reduce(const uint2* __restrict__ tasks, const uint32_t* __restrict__ start,
-              const uint32_t* __restrict__ sorted_r, const unsigned long long* __restrict__ stats,
-              const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
-              double* __restrict__ g, Touched tc, int log2gs) {
+__global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
+k_range_reduce(const unsigned long long* __restrict__ sorted_e,
+               const unsigned long long* __restrict__ stats, int64_t npairs,
+               const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
+               double* __restrict__ g, Touched tc, int log2gs) {
     using V = Vec<VW>;
     using VT = typename V::T;
     extern __shared__ __align__(16) float s_stage[];   // [groups per CTA][L]
-    const int64_t ntasks = (int64_t)stats[2];
+    const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
+    const int64_t ntasks = (total + kPiece - 1) / kPiece;
     const int lane = threadIdx.x & 31;
     const int gs = 1 << log2gs;
     const int lg = lane & (gs - 1);
@@ -206,27 +219,50 @@ k_task_reduce(const uint2* __restrict__ tasks, const uint32_t* __restrict__ star
     const unsigned gmask = (gs == 32) ? 0xffffffffu
                                       : (((1u << gs) - 1u) << ((lane >> log2gs) << log2gs));
     const int64_t gstride = (int64_t)gridDim.x * kWarps * gpw;
+    float s[KC][VW], c[KC][VW];
+
+    auto flush = [&](uint32_t x) {
+#pragma unroll
+        for (int k = 0; k < KC; ++k) {
+            const int col = (lg + k * gs) * VW;
+#pragma unroll
+            for (int i = 0; i < VW; ++i) {
+                if (col + i < L) stage[col + i] = s[k][i];
+                s[k][i] = c[k][i] = 0.f;
+            }
+        }
+        __syncwarp(gmask);
+        double* base = g + (int64_t)x * G;
+        for (int z = lg; z < L; z += gs) {
+            const float val = stage[z];
+            if (val != 0.f) red_add_f64(base + z, widen(val));
+        }
+        if (tc.bitmap && lg == 0) mark_touched(tc, x);
+        __syncwarp(gmask);
+    };
+
     for (int64_t t = (int64_t)blockIdx.x * kWarps * gpw + grp; t < ntasks; t += gstride) {
-        const uint2 tk = __ldg(tasks + t);
-        const uint32_t x = tk.x;
-        const uint32_t e0 = __ldg(start + x) + tk.y * kPiece;
-        const uint32_t eb = __ldg(start + x + 1);
-        const uint32_t e1 = (e0 + kPiece < eb) ? e0 + kPiece : eb;
-        float s[KC][VW], c[KC][VW];
+        const int64_t e0 = t * kPiece;
+        const int64_t e1 = (e0 + kPiece < total) ? e0 + kPiece : total;
 #pragma unroll
         for (int k = 0; k < KC; ++k)
 #pragma unroll
             for (int i = 0; i < VW; ++i) s[k][i] = c[k][i] = 0.f;
-        for (uint32_t e = e0; e < e1; e += kRU) {
+        uint32_t cur = (uint32_t)(__ldg(sorted_e + e0) >> 32);
+        for (int64_t e = e0; e < e1; e += kRU) {
+            uint32_t xs[kRU];
             VT v[kRU][KC];
 #pragma unroll
             for (int u = 0; u < kRU; ++u) {
+                xs[u] = kBad;
 #pragma unroll
                 for (int k = 0; k < KC; ++k)
 #pragma unroll
                     for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
                 if (e + u < e1) {
-                    const uint32_t r = __ldg(sorted_r + e + u);
+                    const unsigned long long ent = __ldg(sorted_e + e + u);
+                    xs[u] = (uint32_t)(ent >> 32);
+                    const uint32_t r = (uint32_t)ent;
                     const uint32_t row = JPOW2 ? (r >> log2J) : r / (uint32_t)J;
                     const int j = (int)(r - row * (uint32_t)J);
                     const int Lj = (d - j * Z) < Z ? (d - j * Z) : Z;
@@ -239,29 +275,19 @@ k_task_reduce(const uint2* __restrict__ tasks, const uint32_t* __restrict__ star
                 }
             }
 #pragma unroll
-            for (int u = 0; u < kRU; ++u)
+            for (int u = 0; u < kRU; ++u) {
+                if (xs[u] == kBad) break;
+                if (xs[u] != cur) {
+                    flush(cur);
+                    cur = xs[u];
+                }
 #pragma unroll
                 for (int k = 0; k < KC; ++k)
 #pragma unroll
                     for (int i = 0; i < VW; ++i) kahan_add(s[k][i], c[k][i], V::get(v[u][k], i));
+            }
         }
-        // transpose through shared memory so that each fp64 reduction
-        // instruction covers consecutive elements
-#pragma unroll
-        for (int k = 0; k < KC; ++k) {
-            const int col = (lg + k * gs) * VW;
-#pragma unroll
-            for (int i = 0; i < VW; ++i)
-                if (col + i < L) stage[col + i] = s[k][i];
-        }
-        __syncwarp(gmask);
-        double* base = g + (int64_t)x * G;
-        for (int z = lg; z < L; z += gs) {
-            const float val = stage[z];
-            if (val != 0.f) red_add_f64(base + z, (double)val);
-        }
-        if (tc.bitmap && lg == 0) mark_touched(tc, x);
-        __syncwarp(gmask);
+        flush(cur);
     }
 }
 
@@ -272,18 +298,16 @@ cudaError_t reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* go
     const int log2J = (p.J & (p.J - 1)) == 0 ? ceil_log2(p.J) : -1;
     const int gpc = kWarps * (32 >> log2gs);
     const size_t smem = sizeof(float) * (size_t)gpc * (size_t)p.L;
-    // tasks <= valid pairs <= npairs; the exact count is read on the device
-    const int64_t work_blocks = (npairs + gpc - 1) / gpc;
+    const int64_t ntasks = (npairs + kPiece - 1) / kPiece;   // upper bound
+    const int64_t work_blocks = (ntasks + gpc - 1) / gpc;
     if (log2J >= 0) {
-        const int grid = grid_for(k_task_reduce<VW, KC, true>, sm_count, work_blocks, smem);
-        k_task_reduce<VW, KC, true><<<grid, kThreads, smem, st>>>(
-            sb.tasks, sb.start, sb.sorted_r, sb.stats, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, tc,
-            log2gs);
+        const int grid = grid_for(k_range_reduce<VW, KC, true>, sm_count, work_blocks, smem);
+        k_range_reduce<VW, KC, true><<<grid, kThreads, smem, st>>>(
+            sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, tc, log2gs);
     } else {
-        const int grid = grid_for(k_task_reduce<VW, KC, false>, sm_count, work_blocks, smem);
-        k_task_reduce<VW, KC, false><<<grid, kThreads, smem, st>>>(
-            sb.tasks, sb.start, sb.sorted_r, sb.stats, gout, p.d, p.Z, p.J, 0, p.L, p.G, g, tc,
-            log2gs);
+        const int grid = grid_for(k_range_reduce<VW, KC, false>, sm_count, work_blocks, smem);
+        k_range_reduce<VW, KC, false><<<grid, kThreads, smem, st>>>(
+            sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, 0, p.L, p.G, g, tc, log2gs);
     }
     return cudaGetLastError();
 }
@@ -292,20 +316,17 @@ cudaError_t reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* go
 
 int64_t sorted_scan_blocks(int64_t R) { return (R + kScanChunk - 1) / kScanChunk; }
 
-int64_t sorted_max_tasks(int64_t R, int64_t npairs) {
-    return (R < npairs ? R : npairs) + npairs / kPiece + 1;
-}
+
 
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, cudaStream_t st) {
     const int64_t nblk = sorted_scan_blocks(R);
-    k_scan_reduce<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.btask, sb.bnz);
+    k_scan_reduce<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.bnz);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_scan_top<<<1, kScanThreads, 0, st>>>(sb.bsum, sb.btask, sb.bnz, nblk, sb.stats);
+    k_scan_top<<<1, kScanThreads, 0, st>>>(sb.bsum, sb.bnz, nblk, sb.stats);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_scan_apply<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.btask, sb.start,
-                                                          sb.tasks);
+    k_scan_apply<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.start);
     return cudaGetLastError();
 }
 
@@ -314,7 +335,7 @@ cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J
     const int log2J = (J & (J - 1)) == 0 ? ceil_log2(J) : -1;
     const int grid = grid_for(k_sort_scatter, sm_count, (npairs + kThreads - 1) / kThreads);
     k_sort_scatter<<<grid, kThreads, 0, st>>>(sb.pair_x, npairs, sb.q_row, J, log2J, sb.start,
-                                              sb.cnt, sb.sorted_r);
+                                              sb.cnt, sb.sorted_e);
     return cudaGetLastError();
 }
 

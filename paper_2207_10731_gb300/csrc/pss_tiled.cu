@@ -1,7 +1,8 @@
 // Tiled forward (hash + gather + sum-pool) and backward scatter kernels.
 //
-// A CTA takes a TILE of `tb` consecutive bags of one table (bag slots
-// t*B + b0 .. t*B + b0 + tb - 1, so the table id is uniform in the tile):
+// The forward gives each warp its own tile (see k_forward_warp).  The atomic
+// backward scatter gives each CTA a TILE of `tb` consecutive bags of one table
+// (bag slots t*B + b0 .. t*B + b0 + tb - 1, so the table id is uniform):
 //   stage:  the tile's offsets go to shared memory; then every (id, chunk)
 //           pair of the tile is hashed ONCE, by one thread, into a shared
 //           array of block buckets x (loc = G*x).  Long tiles are staged in
@@ -23,7 +24,8 @@
 namespace pss {
 namespace {
 
-constexpr int kU = 4;            // ids in flight per group
+constexpr int kU = 4;            // ids in flight per group (the multi-id path sums them as a tree)
+static_assert(kU == 4, "the multi-id forward sums kU = 4 values per round as a tree");
 constexpr int kBagsPerGroup = 16;
 
 template <typename XT>
@@ -95,42 +97,94 @@ __device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t*
 }
 
 // ---------------------------------------------------------------------------
+// Forward.  Each WARP owns a tile of `wb` consecutive bags of one table and
+// stages it in its own slice of shared memory, so warps never wait for each
+// other (no CTA-wide barrier): the lanes hash the tile's (id, chunk) pairs
+// 32 at a time, then the lane groups gather and sum-pool their bags.
+constexpr int kWarpPairs = 512;   // staged pairs per warp and round
+
+// Hash the pairs [0, nq*J) of ids qc0.. into s_x (warp-cooperative); emits
+// buckets / counts for the sorted backward when asked.  Counts of equal
+// buckets within the 32 pairs of a round are merged before the atomic.
+template <typename XT>
+__device__ __forceinline__ void warp_stage(const DevParams& p, const int64_t* __restrict__ idx,
+                                           int t, uint64_t card, int64_t qc0, int nq, XT* s_x,
+                                           DevError* err, uint32_t* __restrict__ pair_x,
+                                           uint32_t* __restrict__ cnt, int lane) {
+    const int npairs = nq * p.J;
+    const bool jpow2 = (p.J & (p.J - 1)) == 0;
+    const int log2J = 31 - __clz(p.J);
+    for (int base = 0; base < npairs; base += 32) {
+        const int k = base + lane;
+        XT x = Invalid<XT>::v;
+        if (k < npairs) {
+            const int qi = jpow2 ? (k >> log2J) : k / p.J;
+            const int j = k - qi * p.J;
+            const int64_t q = qc0 + qi;
+            const int64_t id = __ldg(idx + q);
+            if ((uint64_t)id < card) x = (XT)hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
+            else if (j == 0) record_bad_id(err, q);
+            s_x[k] = x;
+            if (pair_x) pair_x[qc0 * p.J + k] = (uint32_t)x;
+        }
+        if (cnt) {
+            const unsigned peers = __match_any_sync(0xffffffffu, (uint32_t)x);
+            if (x != Invalid<XT>::v && lane == __ffs(peers) - 1)
+                atomicAdd(cnt + (uint64_t)x, (uint32_t)__popc(peers));
+        }
+    }
+    __syncwarp();
+}
+
 template <int VW, int KC, typename XT>
-__global__ void __launch_bounds__(kThreads)
-k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
-                const int64_t* __restrict__ off, int64_t B, const float* __restrict__ w,
-                float* __restrict__ out, DevError* err, uint32_t* __restrict__ pair_x,
-                uint32_t* __restrict__ q_row, uint32_t* __restrict__ cnt, int log2gs,
-                TileGeom tg) {
+__global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
+k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
+               const int64_t* __restrict__ off, int64_t B, const float* __restrict__ w,
+               float* __restrict__ out, DevError* err, uint32_t* __restrict__ pair_x,
+               uint32_t* __restrict__ q_row, uint32_t* __restrict__ cnt, int log2gs, int wb,
+               int tiles_per_table) {
     using V = Vec<VW>;
     using VT = typename V::T;
     extern __shared__ __align__(16) unsigned char smem[];
-    int64_t* s_off = reinterpret_cast<int64_t*>(smem);
-    XT* s_x = reinterpret_cast<XT*>(s_off + tg.tb + 1);
-    __shared__ int s_bad;
-
+    const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    int64_t* s_off = reinterpret_cast<int64_t*>(smem) + warp * (wb + 1);
+    XT* s_x = reinterpret_cast<XT*>(reinterpret_cast<int64_t*>(smem) + kWarps * (wb + 1)) +
+              warp * kWarpPairs;
     const int gs = 1 << log2gs;
     const int lg = lane & (gs - 1);
-    const int grp = (threadIdx.x >> 5) * (32 >> log2gs) + (lane >> log2gs);
+    const int g = lane >> log2gs;
+    const int bpg = wb >> (5 - log2gs);      // bags per group
     const Cols<VW, KC> col(p, lg, gs);
     const uint64_t G = (uint64_t)p.G;
     const int J = p.J;
-    const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
-    const Touched none{};
+    const int qcw = kWarpPairs / J;          // ids per staging round
+    const int64_t ntiles = (int64_t)p.T * tiles_per_table;
+    const int64_t ostride = (int64_t)p.T * p.d;
 
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-        const int t = (int)(tile / tg.tiles_per_table);
-        const int64_t b0 = (tile - (int64_t)t * tg.tiles_per_table) * tg.tb;
-        const int nb = (int)((B - b0) < tg.tb ? (B - b0) : tg.tb);
+    for (int64_t tile = (int64_t)blockIdx.x * kWarps + warp; tile < ntiles;
+         tile += (int64_t)gridDim.x * kWarps) {
+        // ntiles < 2^31 (checked by the launcher): 32-bit division
+        const int t = (int)((uint32_t)tile / (uint32_t)tiles_per_table);
+        const int64_t b0 = (tile - (int64_t)t * tiles_per_table) * wb;
+        const int nb = (int)((B - b0) < wb ? (B - b0) : wb);
         const int64_t s0 = (int64_t)t * B + b0;
-        const int gb0 = min(grp * kBagsPerGroup, nb);
-        const int gb1 = min(gb0 + kBagsPerGroup, nb);
-        float* obase = out + ((b0 * p.T) + t) * (int64_t)p.d;   // row of bag b0
-        const int64_t ostride = (int64_t)p.T * p.d;               // next bag row
+        float* obase = out + ((b0 * p.T) + t) * (int64_t)p.d;
+        const int gb0 = min(g * bpg, nb);
+        const int gb1 = min(gb0 + bpg, nb);
 
-        bool one_hot = false;
-        if (!stage_offsets(off, s0, nb, nnz, s_off, &s_bad, err, &one_hot)) {
+        for (int i = lane; i <= nb; i += 32) s_off[i] = __ldg(off + s0 + i);
+        __syncwarp();
+        bool bad = false, multi = false;
+        for (int i = lane; i < nb; i += 32) {
+            const int64_t a = s_off[i], c = s_off[i + 1];
+            bad |= (a < 0 || c < a || c > nnz);
+            multi |= (c - a > 1);
+        }
+        bad = __any_sync(0xffffffffu, bad);
+        multi = __any_sync(0xffffffffu, multi);
+        if (bad) {
+            if (lane == 0) record_bad_offsets(err);
             for (int bi = gb0; bi < gb1; ++bi)
 #pragma unroll
                 for (int k = 0; k < KC; ++k) {
@@ -140,21 +194,20 @@ k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                     for (int i = 0; i < VW; ++i) V::set(z, i, 0.f);
                     V::stcs(obase + bi * ostride + col.e[k], z);
                 }
-            __syncthreads();
+            __syncwarp();
             continue;
         }
         const uint64_t card = (uint64_t)__ldg(p.cards + t);
         const int64_t qa = s_off[0], qb = s_off[nb];
-        if (one_hot && qb - qa <= tg.qc) {
-            // every bag holds at most one id: no accumulation, one load per bag
-            stage_buckets<XT, false>(p, idx, t, card, qa, (int)(qb - qa), s_x, err, none, pair_x,
-                                     cnt);
-            __syncthreads();
-            for (int b = gb0; b < gb1; b += kU) {
+
+        if (!multi && qb - qa <= qcw) {
+            // every bag holds at most one id: one load per bag, no accumulation
+            warp_stage<XT>(p, idx, t, card, qa, (int)(qb - qa), s_x, err, pair_x, cnt, lane);
+            for (int bb0 = gb0; bb0 < gb1; bb0 += kU) {
                 VT v[kU][KC];
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
-                    const int bb = b + u;
+                    const int bb = bb0 + u;
                     int64_t q = -1;
                     if (bb < gb1 && s_off[bb + 1] > s_off[bb]) q = s_off[bb];
 #pragma unroll
@@ -168,86 +221,94 @@ k_forward_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                     }
                     if (q >= 0 && q_row && lg == 0) q_row[q] = (uint32_t)((b0 + bb) * p.T + t);
                 }
+                float* orow = obase + bb0 * ostride;
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
-                    const int bb = b + u;
-                    if (bb >= gb1) break;
-                    float* orow = obase + bb * ostride;
+                    if (bb0 + u >= gb1) break;
 #pragma unroll
                     for (int k = 0; k < KC; ++k)
                         if (col.v[k]) V::stcs(orow + col.e[k], v[u][k]);
+                    orow += ostride;
                 }
             }
-            __syncthreads();
+            __syncwarp();
             continue;
         }
-        const int64_t gq0 = s_off[gb0], gq1 = s_off[gb1];
-        int bi = gb0;
-        int64_t qend = (gb0 < gb1) ? s_off[gb0 + 1] : 0;
-        float acc[KC][VW], cmp[KC][VW];
-#pragma unroll
-        for (int k = 0; k < KC; ++k)
-#pragma unroll
-            for (int i = 0; i < VW; ++i) acc[k][i] = cmp[k][i] = 0.f;
 
-        auto flush = [&]() {
-            float* orow = obase + bi * ostride;
+        // general bags: the whole warp takes one bag at a time; its ng lane
+        // groups add ng consecutive ids of the bag in parallel, kU steps per
+        // round.  A round's kU values are summed as a tree and added to the
+        // running sum with compensation (Kahan); at the end of the bag the
+        // groups' sums are merged the same way and group 0 stores the row.
+        const int ng = 32 >> log2gs;
+        int64_t sw0 = 0, sw1 = 0;        // ids staged in s_x: [sw0, sw1)
+        for (int bi = 0; bi < nb; ++bi) {
+            const int64_t a = s_off[bi], c = s_off[bi + 1];
+            float acc[KC][VW], cmp[KC][VW];
 #pragma unroll
-            for (int k = 0; k < KC; ++k) {
-                if (!col.v[k]) continue;
-                VT o;
+            for (int k = 0; k < KC; ++k)
 #pragma unroll
-                for (int i = 0; i < VW; ++i) {
-                    V::set(o, i, acc[k][i]);
-                    acc[k][i] = cmp[k][i] = 0.f;
+                for (int i = 0; i < VW; ++i) acc[k][i] = cmp[k][i] = 0.f;
+            const uint32_t row = (uint32_t)((b0 + bi) * p.T + t);
+            for (int64_t q = a; q < c;) {
+                if (q >= sw1) {
+                    sw0 = q;
+                    sw1 = (qb - q) < qcw ? qb : q + qcw;
+                    warp_stage<XT>(p, idx, t, card, sw0, (int)(sw1 - sw0), s_x, err, pair_x, cnt,
+                                   lane);
                 }
-                V::stcs(orow + col.e[k], o);
-            }
-        };
-
-        for (int64_t qc0 = qa; qc0 < qb; qc0 += tg.qc) {
-            const int nq = (int)((qb - qc0) < tg.qc ? (qb - qc0) : tg.qc);
-            stage_buckets<XT, false>(p, idx, t, card, qc0, nq, s_x, err, none, pair_x, cnt);
-            __syncthreads();
-            const int64_t qlo = gq0 > qc0 ? gq0 : qc0;
-            const int64_t qhi = gq1 < qc0 + nq ? gq1 : qc0 + nq;
-            for (int64_t q = qlo; q < qhi; q += kU) {
-                VT v[kU][KC];
+                const int64_t qend = c < sw1 ? c : sw1;
+                for (int64_t qs = q; qs < qend; qs += (int64_t)kU * ng) {
+                    VT v[kU][KC];
 #pragma unroll
-                for (int u = 0; u < kU; ++u) {
+                    for (int u = 0; u < kU; ++u) {
+                        const int64_t qq = qs + (int64_t)u * ng + g;
 #pragma unroll
-                    for (int k = 0; k < KC; ++k) {
+                        for (int k = 0; k < KC; ++k) {
 #pragma unroll
-                        for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
-                        if (q + u < qhi && col.v[k]) {
-                            const XT x = s_x[(int)(q + u - qc0) * J + col.j[k]];
-                            if (x != Invalid<XT>::v) v[u][k] = V::ldg(w + G * (uint64_t)x + col.z[k]);
+                            for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
+                            if (qq < qend && col.v[k]) {
+                                const XT x = s_x[(int)(qq - sw0) * J + col.j[k]];
+                                if (x != Invalid<XT>::v) v[u][k] = V::ldg(w + G * (uint64_t)x + col.z[k]);
+                            }
                         }
+                        if (qq < qend && q_row && lg == 0) q_row[qq] = row;
                     }
-                }
-#pragma unroll
-                for (int u = 0; u < kU; ++u) {
-                    if (q + u >= qhi) break;
-                    while (q + u >= qend) {
-                        flush();
-                        ++bi;
-                        qend = s_off[bi + 1];
-                    }
-                    if (q_row && lg == 0) q_row[q + u] = (uint32_t)((b0 + bi) * p.T + t);
 #pragma unroll
                     for (int k = 0; k < KC; ++k)
 #pragma unroll
-                        for (int i = 0; i < VW; ++i) kahan_add(acc[k][i], cmp[k][i], V::get(v[u][k], i));
+                        for (int i = 0; i < VW; ++i) {
+                            const float s01 = V::get(v[0][k], i) + V::get(v[1][k], i);
+                            const float s23 = V::get(v[2][k], i) + V::get(v[3][k], i);
+                            kahan_add(acc[k][i], cmp[k][i], s01 + s23);
+                        }
+                }
+                q = qend;
+            }
+            for (int o = gs; o < 32; o <<= 1) {
+#pragma unroll
+                for (int k = 0; k < KC; ++k)
+#pragma unroll
+                    for (int i = 0; i < VW; ++i) {
+                        const float os = __shfl_xor_sync(0xffffffffu, acc[k][i], o);
+                        const float oc = __shfl_xor_sync(0xffffffffu, cmp[k][i], o);
+                        kahan_add(acc[k][i], cmp[k][i], os);
+                        kahan_add(acc[k][i], cmp[k][i], -oc);
+                    }
+            }
+            if (g == 0) {
+                float* orow = obase + bi * ostride;
+#pragma unroll
+                for (int k = 0; k < KC; ++k) {
+                    if (!col.v[k]) continue;
+                    VT o;
+#pragma unroll
+                    for (int i = 0; i < VW; ++i) V::set(o, i, acc[k][i] - cmp[k][i]);
+                    V::stcs(orow + col.e[k], o);
                 }
             }
-            __syncthreads();
         }
-        // the current bag and any trailing empty bags
-        while (bi < gb1) {
-            flush();
-            ++bi;
-        }
-        __syncthreads();
+        __syncwarp();
     }
 }
 
@@ -372,12 +433,17 @@ cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* id
                      const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
                      uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt, int sm_count,
                      cudaStream_t st) {
-    const TileGeom tg = tile_geom(p, lay, B, sizeof(XT));
-    const size_t smem = tile_smem(tg, p, sizeof(XT));
-    const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
-    const int grid = grid_for(k_forward_tiled<VW, KC, XT>, sm_count, ntiles, smem);
-    k_forward_tiled<VW, KC, XT><<<grid, kThreads, smem, st>>>(p, idx, nnz, off, B, w, out, err,
-                                                              pair_x, q_row, cnt, lay.log2gs, tg);
+    const int wb = (32 >> lay.log2gs) * kBagsPerGroup;      // bags per warp tile
+    const int tpt = (int)((B + wb - 1) / wb);
+    const size_t smem = (size_t)kWarps * ((size_t)(wb + 1) * sizeof(int64_t) +
+                                          (size_t)kWarpPairs * sizeof(XT));
+    const int64_t ntiles = (int64_t)p.T * tpt;
+    if (ntiles >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
+    const int grid = grid_for(k_forward_warp<VW, KC, XT>, sm_count, (ntiles + kWarps - 1) / kWarps,
+                              smem);
+    k_forward_warp<VW, KC, XT><<<grid, kThreads, smem, st>>>(p, idx, nnz, off, B, w, out, err,
+                                                             pair_x, q_row, cnt, lay.log2gs, wb,
+                                                             tpt);
     return cudaGetLastError();
 }
 
