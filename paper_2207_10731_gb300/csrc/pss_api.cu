@@ -226,9 +226,9 @@ pss_status ensure_touched(pss_handle* h, int64_t pairs, cudaStream_t st) {
 bool use_touched(const pss_handle* h, int64_t pairs) {
     if (h->update_mode == PSS_UPDATE_DENSE) return false;
     if (h->update_mode == PSS_UPDATE_TOUCHED) return true;
-    // dense pass reads/writes ~5 words per element of M; the touched pass
-    // costs ~5 words per element of each distinct block plus the marking.
-    return h->dp.M > 2 * pairs * (int64_t)h->dp.L;
+    // the dense pass touches every element of M once; the touched pass visits
+    // at most pairs*L elements at random (measured crossover near M = pairs*L)
+    return h->dp.M > pairs * (int64_t)h->dp.L;
 }
 
 // Largest bucket count for which the sorted path keeps per-bucket counters
@@ -587,7 +587,7 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool touch, c
     poll_stats(h);
     {
         LaunchScope ls(h, PSS_K_SORT, st, 4);
-        PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, st));
+        PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, touch ? &h->touched : nullptr, st));
         PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->sm_count, st));
     }
     if (!h->stats_pending) {

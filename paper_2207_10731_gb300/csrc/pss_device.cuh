@@ -183,14 +183,25 @@ __device__ __forceinline__ bool bag_range(const int64_t* __restrict__ off, int64
 }
 
 
-// Record a distinct block start x in the touched bitmap / list (first marker appends).
-__device__ __forceinline__ void mark_touched(const Touched& tc, uint64_t x) {
-    uint32_t* wp = tc.bitmap + (x >> 5);
-    const uint32_t bit = 1u << (x & 31);
-    if (*reinterpret_cast<volatile uint32_t*>(wp) & bit) return;
-    const uint32_t old = atomicOr(wp, bit);
-    if (!(old & bit)) {
-        const unsigned long long slot = atomicAdd(tc.count, 1ULL);
+// Record distinct block starts in the touched bitmap / list: the lane that
+// sets a bucket's bit first appends it; the appends of a warp share one
+// atomic on the list counter.  All 32 lanes must call this together.
+__device__ __forceinline__ void mark_touched_warp(const Touched& tc, uint64_t x, bool valid,
+                                                  int lane) {
+    bool first = false;
+    if (valid) {
+        uint32_t* wp = tc.bitmap + (x >> 5);
+        const uint32_t bit = 1u << (x & 31);
+        if (!(*reinterpret_cast<volatile uint32_t*>(wp) & bit)) first = !(atomicOr(wp, bit) & bit);
+    }
+    const unsigned m = __ballot_sync(0xffffffffu, first);
+    if (m == 0u) return;
+    const int leader = __ffs(m) - 1;
+    unsigned long long base = 0;
+    if (lane == leader) base = atomicAdd(tc.count, (unsigned long long)__popc(m));
+    base = __shfl_sync(0xffffffffu, base, leader);
+    if (first) {
+        const unsigned long long slot = base + (unsigned long long)__popc(m & ((1u << lane) - 1u));
         if ((int64_t)slot < tc.cap) tc.list[slot] = (int64_t)x;
     }
 }

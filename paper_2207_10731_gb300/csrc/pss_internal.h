@@ -53,7 +53,9 @@ struct SortedBuffers {
     unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j) in bucket order
 };
 int64_t sorted_scan_blocks(int64_t R);
-cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, cudaStream_t st);
+// Bucket starts; with `touched`, also the list / bitmap of non-empty buckets.
+cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
+                               cudaStream_t st);
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
                                   cudaStream_t st);
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,

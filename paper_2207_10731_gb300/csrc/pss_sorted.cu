@@ -88,94 +88,125 @@ k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict_
 
 // Exclusive scan of the chunk sums (one block).  stats[0] = valid pairs,
 // stats[1] = distinct buckets.
+// Exclusive scans of the chunk sums and of the chunk non-empty counts (one
+// block).  stats[0] = valid pairs, stats[1] = distinct buckets, which is also
+// the length of the touched list when one is built.
 __global__ void __launch_bounds__(kScanThreads)
-k_scan_top(uint32_t* __restrict__ bsum, const uint32_t* __restrict__ bnz, int64_t nblk,
-           unsigned long long* __restrict__ stats) {
+k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ bnz, int64_t nblk,
+           unsigned long long* __restrict__ stats, unsigned long long* __restrict__ touched_count) {
     __shared__ uint32_t s_warp[33];
-    __shared__ uint32_t s_carry;
-    __shared__ unsigned long long s_nz[kScanThreads / 32];
-    if (threadIdx.x == 0) s_carry = 0;
+    __shared__ uint32_t s_carry[2];
+    if (threadIdx.x < 2) s_carry[threadIdx.x] = 0;
     __syncthreads();
-    unsigned long long nz = 0;
     for (int64_t b0 = 0; b0 < nblk; b0 += kScanThreads) {
         const int64_t b = b0 + threadIdx.x;
         const bool in = b < nblk;
         const uint32_t v = in ? bsum[b] : 0u;
-        nz += in ? bnz[b] : 0u;
-        uint32_t tot_v;
+        const uint32_t z = in ? bnz[b] : 0u;
+        uint32_t tot_v, tot_z;
         const uint32_t ex_v = block_exclusive_scan(v, s_warp, &tot_v);
-        const uint32_t cv = s_carry;
-        if (in) bsum[b] = cv + ex_v;
+        const uint32_t ex_z = block_exclusive_scan(z, s_warp, &tot_z);
+        const uint32_t cv = s_carry[0], cz = s_carry[1];
+        if (in) {
+            bsum[b] = cv + ex_v;
+            bnz[b] = cz + ex_z;
+        }
         __syncthreads();
-        if (threadIdx.x == 0) s_carry = cv + tot_v;
+        if (threadIdx.x == 0) {
+            s_carry[0] = cv + tot_v;
+            s_carry[1] = cz + tot_z;
+        }
         __syncthreads();
     }
-    for (int o = 16; o > 0; o >>= 1) nz += __shfl_down_sync(0xffffffffu, nz, o);
-    if ((threadIdx.x & 31) == 0) s_nz[threadIdx.x >> 5] = nz;
-    __syncthreads();
     if (threadIdx.x == 0) {
-        unsigned long long total_nz = 0;
-        for (int w = 0; w < (kScanThreads >> 5); ++w) total_nz += s_nz[w];
-        stats[0] = s_carry;
-        stats[1] = total_nz;
+        stats[0] = s_carry[0];
+        stats[1] = s_carry[1];
+        if (touched_count) *touched_count = s_carry[1];
     }
 }
 
-// start[x] = exclusive prefix of cnt; start[R] = total.
+// start[x] = exclusive prefix of cnt; start[R] = total.  With a touched
+// list, the non-empty buckets are listed in order and their bits set.
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_apply(const uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __restrict__ bsum,
-             uint32_t* __restrict__ start) {
+             const uint32_t* __restrict__ bnz, uint32_t* __restrict__ start, Touched tc) {
     __shared__ uint32_t s_warp[33];
     const int64_t base = (int64_t)blockIdx.x * kScanChunk;
     uint32_t c[kScanPerThread];
-    uint32_t sum = 0;
+    uint32_t sum = 0, nz = 0;
 #pragma unroll
     for (int i = 0; i < kScanPerThread; ++i) {
         const int64_t e = base + (int64_t)threadIdx.x * kScanPerThread + i;
         c[i] = (e < R) ? cnt[e] : 0u;
         sum += c[i];
+        nz += (c[i] != 0u);
     }
     uint32_t tot;
     uint32_t run = bsum[blockIdx.x] + block_exclusive_scan(sum, s_warp, &tot);
+    uint32_t zrun = bnz[blockIdx.x] + block_exclusive_scan(nz, s_warp, &tot);
 #pragma unroll
     for (int i = 0; i < kScanPerThread; ++i) {
         const int64_t e = base + (int64_t)threadIdx.x * kScanPerThread + i;
         if (e < R) start[e] = run;
         run += c[i];
         if (e == R - 1) start[R] = run;
+        if (tc.list && c[i] != 0u) {
+            if ((int64_t)zrun < tc.cap) tc.list[zrun] = e;
+            atomicOr(tc.bitmap + (e >> 5), 1u << (e & 31));
+            ++zrun;
+        }
     }
 }
 
 // Slot of every valid pair; cnt counts back down to zero.  Lanes of a warp
-// with the same bucket share one atomic (the leader takes n slots at once).
+// with the same bucket share one atomic (the leader takes n slots at once);
+// each warp keeps kSU such rounds in flight.
+constexpr int kSU = 4;
+
 __global__ void __launch_bounds__(kThreads)
 k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
                int J, int log2J, const uint32_t* __restrict__ start, uint32_t* __restrict__ cnt,
                unsigned long long* __restrict__ sorted_e) {
     const int lane = threadIdx.x & 31;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t p0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); p0 < npairs;
-         p0 += stride) {
-        const int64_t p = p0 + lane;
-        const uint32_t x = (p < npairs) ? __ldg(pair_x + p) : kBad;
-        // loads that do not depend on the slot go first, so they overlap the atomic
-        const uint32_t pp = (uint32_t)p;            // npairs < 2^32 on this path
-        const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
-        const uint32_t j = pp - q * (uint32_t)J;
-        uint32_t row = 0, st0 = 0;
-        if (x != kBad) {
-            row = __ldg(q_row + q);
-            st0 = __ldg(start + x);
+    const int64_t wstride = (int64_t)gridDim.x * blockDim.x * kSU;
+    for (int64_t p0 = ((int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31)) * kSU; p0 < npairs;
+         p0 += wstride) {
+        uint32_t x[kSU], row[kSU], st0[kSU], old[kSU], jj[kSU];
+        unsigned peers[kSU];
+#pragma unroll
+        for (int u = 0; u < kSU; ++u) {
+            const int64_t p = p0 + u * 32 + lane;
+            x[u] = (p < npairs) ? __ldg(pair_x + p) : kBad;
         }
-        const unsigned peers = __match_any_sync(0xffffffffu, x);
-        const int leader = __ffs(peers) - 1;
-        const int rank = __popc(peers & ((1u << lane) - 1u));
-        uint32_t old = 0;
-        if (x != kBad && lane == leader) old = atomicSub(cnt + x, (uint32_t)__popc(peers));
-        old = __shfl_sync(0xffffffffu, old, leader);
-        if (x == kBad) continue;
-        const uint32_t slot = st0 + old - 1u - (uint32_t)rank;
-        sorted_e[slot] = ((unsigned long long)x << 32) | (row * (uint32_t)J + j);
+        // loads that do not depend on the slot go first, so they overlap the atomics
+#pragma unroll
+        for (int u = 0; u < kSU; ++u) {
+            const uint32_t pp = (uint32_t)(p0 + u * 32 + lane);   // npairs < 2^32 on this path
+            const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
+            jj[u] = pp - q * (uint32_t)J;
+            row[u] = 0;
+            st0[u] = 0;
+            if (x[u] != kBad) {
+                row[u] = __ldg(q_row + q);
+                st0[u] = __ldg(start + x[u]);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kSU; ++u) {
+            peers[u] = __match_any_sync(0xffffffffu, x[u]);
+            old[u] = 0;
+            if (x[u] != kBad && lane == __ffs(peers[u]) - 1)
+                old[u] = atomicSub(cnt + x[u], (uint32_t)__popc(peers[u]));
+        }
+#pragma unroll
+        for (int u = 0; u < kSU; ++u) {
+            const int leader = __ffs(peers[u]) - 1;
+            const uint32_t o = __shfl_sync(0xffffffffu, old[u], leader);
+            if (x[u] == kBad) continue;
+            const uint32_t rank = (uint32_t)__popc(peers[u] & ((1u << lane) - 1u));
+            const uint32_t slot = st0[u] + o - 1u - rank;
+            sorted_e[slot] = ((unsigned long long)x[u] << 32) | (row[u] * (uint32_t)J + jj[u]);
+        }
     }
 }
 
@@ -237,7 +268,6 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
             const float val = stage[z];
             if (val != 0.f) red_add_f64(base + z, widen(val));
         }
-        if (tc.bitmap && lg == 0) mark_touched(tc, x);
         __syncwarp(gmask);
     };
 
@@ -248,21 +278,31 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
         for (int k = 0; k < KC; ++k)
 #pragma unroll
             for (int i = 0; i < VW; ++i) s[k][i] = c[k][i] = 0.f;
-        uint32_t cur = (uint32_t)(__ldg(sorted_e + e0) >> 32);
+        constexpr unsigned long long kNone = (unsigned long long)kBad << 32;
+        // entries of the next block are loaded one block ahead
+        unsigned long long nxt[kRU];
+#pragma unroll
+        for (int u = 0; u < kRU; ++u) nxt[u] = (e0 + u < e1) ? __ldg(sorted_e + e0 + u) : kNone;
+        uint32_t cur = (uint32_t)(nxt[0] >> 32);
         for (int64_t e = e0; e < e1; e += kRU) {
             uint32_t xs[kRU];
             VT v[kRU][KC];
+            unsigned long long ent[kRU];
 #pragma unroll
             for (int u = 0; u < kRU; ++u) {
-                xs[u] = kBad;
+                ent[u] = nxt[u];
+                const int64_t en = e + kRU + u;
+                nxt[u] = (en < e1) ? __ldg(sorted_e + en) : kNone;
+            }
+#pragma unroll
+            for (int u = 0; u < kRU; ++u) {
+                xs[u] = (uint32_t)(ent[u] >> 32);
 #pragma unroll
                 for (int k = 0; k < KC; ++k)
 #pragma unroll
                     for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
-                if (e + u < e1) {
-                    const unsigned long long ent = __ldg(sorted_e + e + u);
-                    xs[u] = (uint32_t)(ent >> 32);
-                    const uint32_t r = (uint32_t)ent;
+                if (xs[u] != kBad) {
+                    const uint32_t r = (uint32_t)ent[u];
                     const uint32_t row = JPOW2 ? (r >> log2J) : r / (uint32_t)J;
                     const int j = (int)(r - row * (uint32_t)J);
                     const int Lj = (d - j * Z) < Z ? (d - j * Z) : Z;
@@ -318,15 +358,17 @@ int64_t sorted_scan_blocks(int64_t R) { return (R + kScanChunk - 1) / kScanChunk
 
 
 
-cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, cudaStream_t st) {
+cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
+                               cudaStream_t st) {
     const int64_t nblk = sorted_scan_blocks(R);
+    const Touched tc = touched ? *touched : Touched{};
     k_scan_reduce<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.bnz);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_scan_top<<<1, kScanThreads, 0, st>>>(sb.bsum, sb.bnz, nblk, sb.stats);
+    k_scan_top<<<1, kScanThreads, 0, st>>>(sb.bsum, sb.bnz, nblk, sb.stats, tc.count);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    k_scan_apply<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.start);
+    k_scan_apply<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.bnz, sb.start, tc);
     return cudaGetLastError();
 }
 

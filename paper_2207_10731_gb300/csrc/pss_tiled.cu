@@ -68,31 +68,29 @@ __device__ __forceinline__ bool stage_offsets(const int64_t* __restrict__ off, i
     return !(flags & 1);
 }
 
-// Hash every (id, chunk) pair of ids [qc0, qc0 + nq) of table t into s_x.
+// Hash every (id, chunk) pair of ids [qc0, qc0 + nq) of table t into s_x
+// (CTA-cooperative; used by the atomic backward scatter).  With TOUCH every
+// distinct bucket is also recorded in the touched bitmap / list, with one
+// list-counter atomic per warp.
 template <typename XT, bool TOUCH>
 __device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t* __restrict__ idx,
                                               int t, uint64_t card, int64_t qc0, int nq, XT* s_x,
-                                              DevError* err, const Touched& tc,
-                                              uint32_t* __restrict__ pair_x = nullptr,
-                                              uint32_t* __restrict__ cnt = nullptr) {
+                                              DevError* err, const Touched& tc) {
     const int npairs = nq * p.J;
-    for (int k = threadIdx.x; k < npairs; k += kThreads) {
-        const int qi = k / p.J;
-        const int j = k - qi * p.J;
-        const int64_t q = qc0 + qi;
-        const int64_t id = __ldg(idx + q);
-        XT x;
-        if ((uint64_t)id >= card) {
-            x = Invalid<XT>::v;
-            if (j == 0) record_bad_id(err, q);
-        } else {
-            const uint64_t b = hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
-            x = (XT)b;
-            if (TOUCH) mark_touched(tc, b);
-            if (cnt) atomicAdd(cnt + b, 1u);
+    const int lane = threadIdx.x & 31;
+    for (int base = threadIdx.x & ~31; base < npairs; base += kThreads) {   // warp-uniform
+        const int k = base + lane;
+        XT x = Invalid<XT>::v;
+        if (k < npairs) {
+            const int qi = k / p.J;
+            const int j = k - qi * p.J;
+            const int64_t q = qc0 + qi;
+            const int64_t id = __ldg(idx + q);
+            if ((uint64_t)id < card) x = (XT)hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
+            else if (j == 0) record_bad_id(err, q);
+            s_x[k] = x;
         }
-        s_x[k] = x;
-        if (pair_x) pair_x[qc0 * p.J + k] = (uint32_t)x;
+        if (TOUCH) mark_touched_warp(tc, (uint64_t)x, x != Invalid<XT>::v, lane);
     }
 }
 
@@ -126,6 +124,45 @@ __device__ __forceinline__ void warp_stage(const DevParams& p, const int64_t* __
             else if (j == 0) record_bad_id(err, q);
             s_x[k] = x;
             if (pair_x) pair_x[qc0 * p.J + k] = (uint32_t)x;
+        }
+        if (cnt) {
+            const unsigned peers = __match_any_sync(0xffffffffu, (uint32_t)x);
+            if (x != Invalid<XT>::v && lane == __ffs(peers) - 1)
+                atomicAdd(cnt + (uint64_t)x, (uint32_t)__popc(peers));
+        }
+    }
+    __syncwarp();
+}
+
+// One-id tiles: stage by BAG.  s_x[bb*J + j] is the bucket of chunk j of the
+// id of bag bb (Invalid for an empty bag or a bad id), so the gather needs no
+// offsets; the id's output row is written here too.
+template <typename XT>
+__device__ __forceinline__ void warp_stage_bags(const DevParams& p, const int64_t* __restrict__ idx,
+                                                int t, uint64_t card, const int64_t* s_off, int nb,
+                                                XT* s_x, DevError* err,
+                                                uint32_t* __restrict__ pair_x,
+                                                uint32_t* __restrict__ q_row,
+                                                uint32_t* __restrict__ cnt, uint32_t row0,
+                                                int lane) {
+    const int npairs = nb * p.J;
+    const bool jpow2 = (p.J & (p.J - 1)) == 0;
+    const int log2J = 31 - __clz(p.J);
+    for (int base = 0; base < npairs; base += 32) {
+        const int k = base + lane;
+        XT x = Invalid<XT>::v;
+        if (k < npairs) {
+            const int bb = jpow2 ? (k >> log2J) : k / p.J;
+            const int j = k - bb * p.J;
+            const int64_t q = s_off[bb];
+            if (s_off[bb + 1] > q) {
+                const int64_t id = __ldg(idx + q);
+                if ((uint64_t)id < card) x = (XT)hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
+                else if (j == 0) record_bad_id(err, q);
+                if (pair_x) pair_x[q * p.J + j] = (uint32_t)x;
+                if (q_row && j == 0) q_row[q] = row0 + (uint32_t)bb * (uint32_t)p.T;
+            }
+            s_x[k] = x;
         }
         if (cnt) {
             const unsigned peers = __match_any_sync(0xffffffffu, (uint32_t)x);
@@ -200,35 +237,33 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
         const uint64_t card = (uint64_t)__ldg(p.cards + t);
         const int64_t qa = s_off[0], qb = s_off[nb];
 
-        if (!multi && qb - qa <= qcw) {
+        if (!multi && nb * J <= kWarpPairs) {
             // every bag holds at most one id: one load per bag, no accumulation
-            warp_stage<XT>(p, idx, t, card, qa, (int)(qb - qa), s_x, err, pair_x, cnt, lane);
+            warp_stage_bags<XT>(p, idx, t, card, s_off, nb, s_x, err, pair_x, q_row, cnt,
+                                (uint32_t)(b0 * p.T + t), lane);
+            float* orow0 = obase + gb0 * ostride;
             for (int bb0 = gb0; bb0 < gb1; bb0 += kU) {
                 VT v[kU][KC];
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
                     const int bb = bb0 + u;
-                    int64_t q = -1;
-                    if (bb < gb1 && s_off[bb + 1] > s_off[bb]) q = s_off[bb];
 #pragma unroll
                     for (int k = 0; k < KC; ++k) {
 #pragma unroll
                         for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
-                        if (q >= 0 && col.v[k]) {
-                            const XT x = s_x[(int)(q - qa) * J + col.j[k]];
+                        if (bb < gb1 && col.v[k]) {
+                            const XT x = s_x[bb * J + col.j[k]];
                             if (x != Invalid<XT>::v) v[u][k] = V::ldg(w + G * (uint64_t)x + col.z[k]);
                         }
                     }
-                    if (q >= 0 && q_row && lg == 0) q_row[q] = (uint32_t)((b0 + bb) * p.T + t);
                 }
-                float* orow = obase + bb0 * ostride;
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
                     if (bb0 + u >= gb1) break;
 #pragma unroll
                     for (int k = 0; k < KC; ++k)
-                        if (col.v[k]) V::stcs(orow + col.e[k], v[u][k]);
-                    orow += ostride;
+                        if (col.v[k]) V::stcs(orow0 + col.e[k], v[u][k]);
+                    orow0 += ostride;
                 }
             }
             __syncwarp();

@@ -502,6 +502,7 @@ def test_profile_and_launch_counts():
     h, _ = gu.make_pair(w)
     h.set_option(binding.OPT_PROFILE, 1)
     h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_ATOMIC)
+    h.set_option(binding.OPT_UPDATE_MODE, binding.UPDATE_DENSE)
     idx, off = _batch_cuda(w)
     go = gu.cuda(w.grad_out)
     before = h.info()["kernel_launches"]
