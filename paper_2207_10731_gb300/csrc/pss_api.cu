@@ -597,8 +597,7 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool touch, c
         h->stats_pending = true;
     }
     LaunchScope ls(h, PSS_K_REDUCE, st);
-    PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64,
-                                 touch ? &h->touched : nullptr, h->sm_count, st));
+    PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64, h->sm_count, st));
     return PSS_OK;
 }
 

@@ -59,8 +59,7 @@ cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
                                   cudaStream_t st);
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                                 const DevParams& p, double* g, const Touched* touched,
-                                 int sm_count, cudaStream_t st);
+                                 const DevParams& p, double* g, int sm_count, cudaStream_t st);
 
 // Kernel launchers (return the CUDA launch error).  `grid_cap` bounds the
 // grid of grid-stride kernels; 0 lets the launcher decide.

@@ -33,7 +33,9 @@ constexpr uint32_t kBad = 0xffffffffu;
 constexpr int kScanThreads = 1024;
 constexpr int kScanPerThread = 8;
 constexpr int kScanChunk = kScanThreads * kScanPerThread;
-constexpr int kRU = 4;            // entries in flight per group
+constexpr int kRU = 4;            // entries in flight per group (summed as a tree when they
+                                  // all continue the current run)
+static_assert(kRU == 4, "the reduce sums kRU = 4 entries as a tree");
 
 // Block-wide exclusive scan of one value per thread (kScanThreads threads).
 __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s_warp,
@@ -230,12 +232,12 @@ __device__ __forceinline__ double widen(float f) {
 // reduction instruction covers consecutive elements).
 constexpr int64_t kPiece = 64;    // sorted entries per reduce task
 
-template <int VW, int KC, bool JPOW2>
+template <int VW, int KC, bool JPOW2, bool ZDIV>
 __global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
 k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                const unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
-               double* __restrict__ g, Touched tc, int log2gs) {
+               double* __restrict__ g, int log2gs) {
     using V = Vec<VW>;
     using VT = typename V::T;
     extern __shared__ __align__(16) float s_stage[];   // [groups per CTA][L]
@@ -250,15 +252,17 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
     const unsigned gmask = (gs == 32) ? 0xffffffffu
                                       : (((1u << gs) - 1u) << ((lane >> log2gs) << log2gs));
     const int64_t gstride = (int64_t)gridDim.x * kWarps * gpw;
+    int colk[KC];
+#pragma unroll
+    for (int k = 0; k < KC; ++k) colk[k] = (lg + k * gs) * VW;
     float s[KC][VW], c[KC][VW];
 
     auto flush = [&](uint32_t x) {
 #pragma unroll
         for (int k = 0; k < KC; ++k) {
-            const int col = (lg + k * gs) * VW;
 #pragma unroll
             for (int i = 0; i < VW; ++i) {
-                if (col + i < L) stage[col + i] = s[k][i];
+                if (colk[k] + i < L) stage[colk[k] + i] = s[k][i];
                 s[k][i] = c[k][i] = 0.f;
             }
         }
@@ -297,59 +301,318 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
             for (int u = 0; u < kRU; ++u) {
                 xs[u] = (uint32_t)(ent[u] >> 32);
-#pragma unroll
-                for (int k = 0; k < KC; ++k)
-#pragma unroll
-                    for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
+                const uint32_t r = (uint32_t)ent[u];
                 if (xs[u] != kBad) {
-                    const uint32_t r = (uint32_t)ent[u];
-                    const uint32_t row = JPOW2 ? (r >> log2J) : r / (uint32_t)J;
-                    const int j = (int)(r - row * (uint32_t)J);
-                    const int Lj = (d - j * Z) < Z ? (d - j * Z) : Z;
-                    const float* src = gout + (int64_t)row * d + j * Z;
+                    if (ZDIV) {
+                        // Z divides d: chunk r starts at r*Z and is Z long
+                        const float* src = gout + (uint64_t)r * (uint64_t)Z;
 #pragma unroll
-                    for (int k = 0; k < KC; ++k) {
-                        const int col = (lg + k * gs) * VW;
-                        if (col < Lj) v[u][k] = V::ldcs(src + col);
+                        for (int k = 0; k < KC; ++k) {
+                            if (colk[k] < L) v[u][k] = V::ldcs(src + colk[k]);
+                            else
+#pragma unroll
+                                for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
+                        }
+                    } else {
+                        const uint32_t row = JPOW2 ? (r >> log2J) : r / (uint32_t)J;
+                        const int j = (int)(r - row * (uint32_t)J);
+                        const int Lj = (d - j * Z) < Z ? (d - j * Z) : Z;
+                        const float* src = gout + (int64_t)row * d + j * Z;
+#pragma unroll
+                        for (int k = 0; k < KC; ++k) {
+                            if (colk[k] < Lj) v[u][k] = V::ldcs(src + colk[k]);
+                            else
+#pragma unroll
+                                for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
+                        }
                     }
+                } else {
+#pragma unroll
+                    for (int k = 0; k < KC; ++k)
+#pragma unroll
+                        for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
                 }
             }
-#pragma unroll
-            for (int u = 0; u < kRU; ++u) {
-                if (xs[u] == kBad) break;
-                if (xs[u] != cur) {
-                    flush(cur);
-                    cur = xs[u];
-                }
+            if (xs[kRU - 1] == cur) {
+                // the whole block continues the current run (keys are sorted):
+                // a tree sum, then one compensated add
 #pragma unroll
                 for (int k = 0; k < KC; ++k)
 #pragma unroll
-                    for (int i = 0; i < VW; ++i) kahan_add(s[k][i], c[k][i], V::get(v[u][k], i));
+                    for (int i = 0; i < VW; ++i) {
+                        const float a01 = V::get(v[0][k], i) + V::get(v[1][k], i);
+                        const float a23 = V::get(v[2][k], i) + V::get(v[3][k], i);
+                        kahan_add(s[k][i], c[k][i], a01 + a23);
+                    }
+            } else {
+#pragma unroll
+                for (int u = 0; u < kRU; ++u) {
+                    if (xs[u] == kBad) break;
+                    if (xs[u] != cur) {
+                        flush(cur);
+                        cur = xs[u];
+                    }
+#pragma unroll
+                    for (int k = 0; k < KC; ++k)
+#pragma unroll
+                        for (int i = 0; i < VW; ++i)
+                            kahan_add(s[k][i], c[k][i], V::get(v[u][k], i));
+                }
             }
         }
         flush(cur);
     }
 }
 
-template <int VW, int KC>
-cudaError_t reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                        const DevParams& p, double* g, const Touched& tc, int log2gs,
-                        int sm_count, cudaStream_t st) {
+// Reduce for blocks of at least 32 elements: one WARP per task of kPiece
+// sorted entries, lane z owning elements z, z+32, ... of the block, so every
+// branch is warp-uniform and a run's sum goes straight from the lanes to the
+// fp64 accumulator (32 consecutive doubles per instruction).  The task's
+// entries are staged in shared memory with one coalesced load; kWU chunk
+// loads per lane are in flight; a block of kWU entries that continues the
+// current run is summed as a tree and added with compensation once.
+constexpr int kWU = 8;
+static_assert(kWU == 8, "the warp reduce sums kWU = 8 entries as a tree");
+
+template <int KE, bool ZDIV, bool JPOW2>
+__global__ void __launch_bounds__(kThreads)
+k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
+                    const unsigned long long* __restrict__ stats, int64_t npairs,
+                    const float* __restrict__ gout, int d, int Z, int J, int log2J, int L,
+                    int64_t G, double* __restrict__ g) {
+    __shared__ unsigned long long s_ent[kWarps][kPiece];
+    const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
+    const int64_t ntasks = (total + kPiece - 1) / kPiece;
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    unsigned long long* ent = s_ent[warp];
+    const int64_t wstride = (int64_t)gridDim.x * kWarps;
+    constexpr unsigned long long kNone = (unsigned long long)kBad << 32;
+    float s[KE], c[KE];
+    auto flush = [&](uint32_t x) {
+        double* base = g + (int64_t)x * G;
+#pragma unroll
+        for (int k = 0; k < KE; ++k) {
+            const int z = lane + 32 * k;
+            if (z < L && s[k] != 0.f) red_add_f64(base + z, widen(s[k]));
+            s[k] = c[k] = 0.f;
+        }
+    };
+    for (int64_t t = (int64_t)blockIdx.x * kWarps + warp; t < ntasks; t += wstride) {
+        const int64_t e0 = t * kPiece;
+        const int n = (int)((e0 + kPiece < total) ? kPiece : total - e0);
+#pragma unroll
+        for (int h = 0; h < (int)kPiece; h += 32)
+            ent[h + lane] = (h + lane < n) ? __ldg(sorted_e + e0 + h + lane) : kNone;
+        __syncwarp();
+#pragma unroll
+        for (int k = 0; k < KE; ++k) s[k] = c[k] = 0.f;
+        uint32_t cur = (uint32_t)(ent[0] >> 32);
+        for (int b = 0; b < n; b += kWU) {
+            uint32_t xs[kWU];
+            float v[kWU][KE];
+#pragma unroll
+            for (int u = 0; u < kWU; ++u) {
+                const unsigned long long en = ent[b + u < (int)kPiece ? b + u : (int)kPiece - 1];
+                xs[u] = (b + u < n) ? (uint32_t)(en >> 32) : kBad;
+                const uint32_t r = (uint32_t)en;
+                const float* src;
+                int Lj;
+                if (ZDIV) {
+                    src = gout + (uint64_t)r * (uint64_t)Z;
+                    Lj = L;
+                } else {
+                    const uint32_t row = JPOW2 ? (r >> log2J) : r / (uint32_t)J;
+                    const int j = (int)(r - row * (uint32_t)J);
+                    Lj = (d - j * Z) < Z ? (d - j * Z) : Z;
+                    src = gout + (int64_t)row * d + j * Z;
+                }
+#pragma unroll
+                for (int k = 0; k < KE; ++k) {
+                    const int z = lane + 32 * k;
+                    v[u][k] = (xs[u] != kBad && z < Lj) ? __ldcs(src + z) : 0.f;
+                }
+            }
+            if (xs[kWU - 1] == cur) {
+#pragma unroll
+                for (int k = 0; k < KE; ++k) {
+                    const float a = (v[0][k] + v[1][k]) + (v[2][k] + v[3][k]);
+                    const float bsum = (v[4][k] + v[5][k]) + (v[6][k] + v[7][k]);
+                    kahan_add(s[k], c[k], a + bsum);
+                }
+            } else {
+#pragma unroll
+                for (int u = 0; u < kWU; ++u) {
+                    if (xs[u] == kBad) break;
+                    if (xs[u] != cur) {
+                        flush(cur);
+                        cur = xs[u];
+                    }
+#pragma unroll
+                    for (int k = 0; k < KE; ++k) kahan_add(s[k], c[k], v[u][k]);
+                }
+            }
+        }
+        flush(cur);
+        __syncwarp();
+    }
+}
+
+// Reduce for 32-element chunks that tile the rows (Z = 32 dividing d): the
+// upstream-gradient chunks of a warp's task are staged asynchronously into
+// shared memory (cp.async, 16 bytes per lane), kAD - 1 stages of kAS chunks in
+// flight per warp, so the data in flight is bounded by shared memory rather
+// than registers.  Lane z then sums element z of each chunk (compensated; a
+// stage that continues the current run is summed as a tree first) and adds
+// every run's sum once into the fp64 accumulator.
+constexpr int kAS = 8;          // chunks per stage
+constexpr int kAD = 4;          // ring slots (kAD - 1 stages in flight)
+constexpr int kAPiece = 128;    // sorted entries per task
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" :: "r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;\n" :: "n"(N) : "memory");
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_async_reduce(const unsigned long long* __restrict__ sorted_e,
+               const unsigned long long* __restrict__ stats, int64_t npairs,
+               const float* __restrict__ gout, int64_t G, double* __restrict__ g) {
+    __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
+    __shared__ unsigned long long s_ent[kWarps][kAPiece];
+    const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
+    const int64_t ntasks = (total + kAPiece - 1) / kAPiece;
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    unsigned long long* ent = s_ent[warp];
+    const int64_t wstride = (int64_t)gridDim.x * kWarps;
+    constexpr unsigned long long kNone = (unsigned long long)kBad << 32;
+    float sum = 0.f, comp = 0.f;
+    auto flush = [&](uint32_t x) {
+        if (sum != 0.f) red_add_f64(g + (int64_t)x * G + lane, widen(sum));
+        sum = comp = 0.f;
+    };
+    for (int64_t t = (int64_t)blockIdx.x * kWarps + warp; t < ntasks; t += wstride) {
+        const int64_t e0 = t * kAPiece;
+        const int n = (int)((e0 + kAPiece < total) ? kAPiece : total - e0);
+#pragma unroll
+        for (int h = 0; h < kAPiece; h += 32)
+            ent[h + lane] = (h + lane < n) ? __ldg(sorted_e + e0 + h + lane) : kNone;
+        __syncwarp();
+        const int nst = (n + kAS - 1) / kAS;
+        // copy stage st (kAS chunks of 128 bytes = 64 pieces of 16 bytes)
+        auto issue = [&](int st) {
+            if (st < nst) {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int pc = lane + 32 * h;
+                    const int i = pc >> 3;
+                    const int part = pc & 7;
+                    const int e = st * kAS + i;
+                    if (e < n) {
+                        const uint32_t r = (uint32_t)ent[e];
+                        cp_async16(&s_ring[warp][st % kAD][i][part * 4],
+                                   gout + (uint64_t)r * 32u + (uint32_t)(part * 4));
+                    }
+                }
+            }
+            cp_async_commit();
+        };
+#pragma unroll
+        for (int st = 0; st < kAD - 1; ++st) issue(st);
+        sum = comp = 0.f;
+        uint32_t cur = (uint32_t)(ent[0] >> 32);
+        for (int st = 0; st < nst; ++st) {
+            issue(st + kAD - 1);
+            cp_async_wait<kAD - 1>();
+            __syncwarp();
+            const float* buf = &s_ring[warp][st % kAD][0][0];
+            uint32_t xs[kAS];
+            float v[kAS];
+#pragma unroll
+            for (int i = 0; i < kAS; ++i) {
+                const int e = st * kAS + i;
+                xs[i] = (e < n) ? (uint32_t)(ent[e] >> 32) : kBad;
+                v[i] = (e < n) ? buf[i * 32 + lane] : 0.f;
+            }
+            if (xs[kAS - 1] == cur) {
+                const float a = (v[0] + v[1]) + (v[2] + v[3]);
+                const float b = (v[4] + v[5]) + (v[6] + v[7]);
+                kahan_add(sum, comp, a + b);
+            } else {
+#pragma unroll
+                for (int i = 0; i < kAS; ++i) {
+                    if (xs[i] == kBad) break;
+                    if (xs[i] != cur) {
+                        flush(cur);
+                        cur = xs[i];
+                    }
+                    kahan_add(sum, comp, v[i]);
+                }
+            }
+            __syncwarp();
+        }
+        flush(cur);
+        cp_async_wait<0>();
+        __syncwarp();
+    }
+}
+
+template <int KE, bool ZDIV, bool JPOW2>
+cudaError_t warp_reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                               const DevParams& p, double* g, int log2J, int sm_count,
+                               cudaStream_t st) {
+    const int64_t ntasks = (npairs + kPiece - 1) / kPiece;   // upper bound
+    const int grid = grid_for(k_warp_range_reduce<KE, ZDIV, JPOW2>, sm_count,
+                              (ntasks + kWarps - 1) / kWarps);
+    k_warp_range_reduce<KE, ZDIV, JPOW2><<<grid, kThreads, 0, st>>>(
+        sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g);
+    return cudaGetLastError();
+}
+
+template <int KE>
+cudaError_t warp_reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                             const DevParams& p, double* g, int sm_count, cudaStream_t st) {
     const int log2J = (p.J & (p.J - 1)) == 0 ? ceil_log2(p.J) : -1;
+    if (p.d % p.Z == 0)
+        return warp_reduce_launch<KE, true, true>(sb, npairs, gout, p, g, 0, sm_count, st);
+    if (log2J >= 0)
+        return warp_reduce_launch<KE, false, true>(sb, npairs, gout, p, g, log2J, sm_count, st);
+    return warp_reduce_launch<KE, false, false>(sb, npairs, gout, p, g, 0, sm_count, st);
+}
+
+template <int VW, int KC, bool JPOW2, bool ZDIV>
+cudaError_t reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                          const DevParams& p, double* g, int log2J, int log2gs, int sm_count,
+                          cudaStream_t st) {
     const int gpc = kWarps * (32 >> log2gs);
     const size_t smem = sizeof(float) * (size_t)gpc * (size_t)p.L;
     const int64_t ntasks = (npairs + kPiece - 1) / kPiece;   // upper bound
     const int64_t work_blocks = (ntasks + gpc - 1) / gpc;
-    if (log2J >= 0) {
-        const int grid = grid_for(k_range_reduce<VW, KC, true>, sm_count, work_blocks, smem);
-        k_range_reduce<VW, KC, true><<<grid, kThreads, smem, st>>>(
-            sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, tc, log2gs);
-    } else {
-        const int grid = grid_for(k_range_reduce<VW, KC, false>, sm_count, work_blocks, smem);
-        k_range_reduce<VW, KC, false><<<grid, kThreads, smem, st>>>(
-            sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, 0, p.L, p.G, g, tc, log2gs);
-    }
+    const int grid = grid_for(k_range_reduce<VW, KC, JPOW2, ZDIV>, sm_count, work_blocks, smem);
+    k_range_reduce<VW, KC, JPOW2, ZDIV><<<grid, kThreads, smem, st>>>(
+        sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, log2gs);
     return cudaGetLastError();
+}
+
+template <int VW, int KC>
+cudaError_t reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                        const DevParams& p, double* g, int log2gs, int sm_count,
+                        cudaStream_t st) {
+    const int log2J = (p.J & (p.J - 1)) == 0 ? ceil_log2(p.J) : -1;
+    if (p.d % p.Z == 0)
+        return reduce_launch<VW, KC, true, true>(sb, npairs, gout, p, g, 0, log2gs, sm_count, st);
+    if (log2J >= 0)
+        return reduce_launch<VW, KC, true, false>(sb, npairs, gout, p, g, log2J, log2gs, sm_count,
+                                                  st);
+    return reduce_launch<VW, KC, false, false>(sb, npairs, gout, p, g, 0, log2gs, sm_count, st);
 }
 
 }  // namespace
@@ -382,15 +645,26 @@ cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J
 }
 
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                                 const DevParams& p, double* g, const Touched* touched,
-                                 int sm_count, cudaStream_t st) {
-    const Touched tc = touched ? *touched : Touched{};
+                                 const DevParams& p, double* g, int sm_count, cudaStream_t st) {
+    // 32-element chunks tiling the rows: asynchronous shared-memory staging
+    if (p.Z == 32 && p.d % 32 == 0 && (((uintptr_t)gout & 15u) == 0)) {
+        const int64_t ntasks = (npairs + kAPiece - 1) / kAPiece;   // upper bound
+        const int grid = grid_for(k_async_reduce, sm_count, (ntasks + kWarps - 1) / kWarps);
+        k_async_reduce<<<grid, kThreads, 0, st>>>(sb.sorted_e, sb.stats, npairs, gout, p.G, g);
+        return cudaGetLastError();
+    }
+    // blocks of 32+ elements: one warp per task, one element per lane
+    if (p.L >= 32) {
+        if (p.L <= 32) return warp_reduce_inst<1>(sb, npairs, gout, p, g, sm_count, st);
+        if (p.L <= 64) return warp_reduce_inst<2>(sb, npairs, gout, p, g, sm_count, st);
+        if (p.L <= 128) return warp_reduce_inst<4>(sb, npairs, gout, p, g, sm_count, st);
+    }
     const bool vec = (p.Z % 4 == 0) && (p.d % 4 == 0) && (((uintptr_t)gout & 15u) == 0);
     const int vw = vec ? 4 : 1;
     const int V = (p.L + vw - 1) / vw;
     const int log2gs = V <= 32 ? ceil_log2(V) : 5;
     const int kc = V <= 32 ? 1 : (1 << ceil_log2((V + 31) / 32));
-#define PSS_RD(VW, KC) return reduce_inst<VW, KC>(sb, npairs, gout, p, g, tc, log2gs, sm_count, st)
+#define PSS_RD(VW, KC) return reduce_inst<VW, KC>(sb, npairs, gout, p, g, log2gs, sm_count, st)
     if (vec) {
         switch (kc) {
             case 1: PSS_RD(4, 1);

@@ -235,7 +235,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
             continue;
         }
         const uint64_t card = (uint64_t)__ldg(p.cards + t);
-        const int64_t qa = s_off[0], qb = s_off[nb];
+        const int64_t qb = s_off[nb];
 
         if (!multi && nb * J <= kWarpPairs) {
             // every bag holds at most one id: one load per bag, no accumulation
