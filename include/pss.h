@@ -267,6 +267,20 @@ pss_status pss_grad_noalloc(const int64_t* table_cardinalities, int32_t num_tabl
                             int64_t B, const float* grad_out, float* grad, int64_t* first_bad,
                             pss_stream stream);
 
+/*
+ * Check of the two conversions of the fp64 gradient accumulation (the paper
+ * has no counterpart: a test hook of this library).  direction 0: out[i] =
+ * the fp32 value in[i] widened exactly to fp64 (in: float[n], out: double[n]);
+ * direction 1: out[i] = fp64 in[i] rounded to the nearest fp32, ties to even
+ * (in: double[n], out: float[n]).  Both are the integer-arithmetic routines the
+ * kernels use, so a caller can compare them bit for bit with IEEE-754
+ * conversions.  `in` and `out` are device buffers owned by the caller.
+ * Asynchronous on `stream`.  Errors: PSS_ERR_INVALID_ARG (direction not 0 or
+ * 1, n < 0, a null or host buffer), PSS_ERR_CUDA.
+ */
+pss_status pss_check_convert(int32_t direction, const void* in, void* out, int64_t n,
+                             pss_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -35,6 +35,7 @@ EXPORTS = [
     "pss_set_state", "pss_compute_locations", "pss_forward", "pss_backward_update",
     "pss_backward_grad", "pss_set_option", "pss_get_option", "pss_get_error", "pss_get_info",
     "pss_get_profile", "pss_reset_profile", "pss_status_string", "pss_grad_noalloc",
+    "pss_check_convert",
 ]
 
 
@@ -89,6 +90,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "pss_reset_profile": [vp],
             "pss_grad_noalloc": [vp, i32, i32, i64, i32, i32, u64, vp, i64, vp, i64, vp, vp, vp,
                                  vp],
+            "pss_check_convert": [i32, vp, vp, i64, vp],
         }
         for name, args in sigs.items():
             fn = getattr(lib, name)

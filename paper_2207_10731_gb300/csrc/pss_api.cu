@@ -314,6 +314,18 @@ pss_status validate_batch(const pss_handle* h, const int64_t* idx, int64_t nnz,
 
 extern "C" {
 
+pss_status pss_check_convert(int32_t direction, const void* in, void* out, int64_t n,
+                             pss_stream stream) {
+    if ((direction != 0 && direction != 1) || n < 0) return PSS_ERR_INVALID_ARG;
+    if (n == 0) return PSS_OK;
+    if (!in || !out || !is_device_ptr(in) || !is_device_ptr(out)) return PSS_ERR_INVALID_ARG;
+    int dev = 0, sms = 0;
+    PSS_TRY(cudaGetDevice(&dev));
+    PSS_TRY(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    PSS_TRY(launch_convert(direction, in, out, n, sms, reinterpret_cast<cudaStream_t>(stream)));
+    return PSS_OK;
+}
+
 const char* pss_status_string(pss_status s) {
     switch (s) {
         case PSS_OK: return "ok";
@@ -536,15 +548,12 @@ pss_status pss_forward(pss_handle* h, const int64_t* indices, int64_t nnz, const
         dout = static_cast<float*>(h->st_out.ptr);
     }
     const bool emit = nbags > 0 && want_sorted(h) && sorted_supported(h, nnz, B);
-    if (emit) {
-        if ((rc = ensure_sorted(h, nnz, st)) != PSS_OK) return rc;
-        PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)h->dp.R, st));
-    }
+    if (emit && (rc = ensure_sorted(h, nnz, st)) != PSS_OK) return rc;
     if (nbags > 0) {
         LaunchScope ls(h, PSS_K_FORWARD, st);
         PSS_TRY(launch_forward(h->dp, layout_for(h, dout), di, nnz, doff, B, h->w, dout, h->err,
                                emit ? h->sb.pair_x : nullptr, emit ? h->sb.q_row : nullptr,
-                               emit ? h->sb.cnt : nullptr, h->sm_count, st));
+                               h->sm_count, st));
     }
     h->batch_emitted = emit;
     if (host_out)
@@ -585,8 +594,10 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool touch, c
     const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
     if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
     poll_stats(h);
+    PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)h->dp.R, st));
     {
-        LaunchScope ls(h, PSS_K_SORT, st, 4);
+        LaunchScope ls(h, PSS_K_SORT, st, 5);
+        PSS_TRY(launch_sorted_count(h->sb, npairs, h->sm_count, st));
         PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, touch ? &h->touched : nullptr, st));
         PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->sm_count, st));
     }

@@ -155,6 +155,33 @@ __device__ __forceinline__ void split_slot(int64_t s, int64_t B, uint64_t Binv, 
     b = (int64_t)r;
 }
 
+// Exact fp32 -> fp64 widening from the IEEE-754 fields, in integer
+// arithmetic only (the FP64 pipe of this part is slow, and a conversion left
+// in a predicated branch would still occupy it): the exponent is re-biased
+// (127 -> 1023) and the 23-bit fraction moved to the top of the 52-bit one; a
+// subnormal input is normalised at its leading one; zeros, infinities and NaNs
+// keep their sign and fraction.
+__device__ __forceinline__ double widen(float f) {
+    const uint32_t u = __float_as_uint(f);
+    const uint64_t sign = (uint64_t)(u & 0x80000000u) << 32;
+    const uint32_t e = (u >> 23) & 0xffu;
+    const uint32_t m = u & 0x7fffffu;
+    uint64_t bits;
+    if (e == 0xffu) {
+        bits = sign | (uint64_t(0x7ff) << 52) | ((uint64_t)m << 29);
+    } else if (e != 0u) {
+        bits = sign | ((uint64_t)(e + 896u) << 52) | ((uint64_t)m << 29);
+    } else if (m == 0u) {
+        bits = sign;
+    } else {
+        // m * 2^-149 with the leading one at bit p: exponent p - 149
+        const int p = 31 - __clz(m);
+        bits = sign | ((uint64_t)(p + 874) << 52) |
+               (((uint64_t)m << (52 - p)) & ((uint64_t(1) << 52) - 1));
+    }
+    return __longlong_as_double((long long)bits);
+}
+
 // Reduction of one VW-wide column into an fp32 or fp64 accumulator.
 template <int VW, typename AT>
 struct Acc;
@@ -164,12 +191,52 @@ struct Acc<VW, float> {
 };
 template <>
 struct Acc<1, double> {
-    static __device__ __forceinline__ void red(double* p, float v) { red_add_f64(p, (double)v); }
+    static __device__ __forceinline__ void red(double* p, float v) { red_add_f64(p, widen(v)); }
 };
+
+// fp64 -> fp32, rounded to nearest (ties to even), in integer arithmetic
+// only (the FP64 pipe of this part is slow).  The 53-bit significand is cut
+// to 24 bits (or, below the normal range, to units of 2^-149) and rounded on
+// the dropped bits; a carry out of the fraction moves into the exponent,
+// which is also how rounding reaches the next binade or infinity.
+__device__ __forceinline__ float narrow(double v) {
+    const uint64_t b = (uint64_t)__double_as_longlong(v);
+    const uint32_t sign = (uint32_t)(b >> 32) & 0x80000000u;
+    const int e = (int)((b >> 52) & 0x7ff);
+    const uint64_t m = b & ((uint64_t(1) << 52) - 1);
+    if (e == 0x7ff)   // infinity, or NaN (kept quiet, top fraction bits kept)
+        return __uint_as_float(sign | 0x7f800000u | (m ? (0x400000u | (uint32_t)(m >> 29)) : 0u));
+    const int ef = e - 1023 + 127;
+    if (ef >= 0xff) return __uint_as_float(sign | 0x7f800000u);
+    if (ef >= 1) {
+        const uint32_t mm = (uint32_t)(m >> 29);
+        const uint64_t rem = m & ((uint64_t(1) << 29) - 1);
+        const uint64_t half = uint64_t(1) << 28;
+        uint32_t r = ((uint32_t)ef << 23) | mm;
+        if (rem > half || (rem == half && (mm & 1u))) r += 1u;
+        return __uint_as_float(sign | r);
+    }
+    if (e == 0) return __uint_as_float(sign);   // below 2^-1022: rounds to zero
+    // significand S = 2^52 + m; the value in units of 2^-149 is S / 2^sh
+    const int sh = 926 - e;                      // >= 30 here
+    if (sh > 54) return __uint_as_float(sign);
+    const uint64_t S = (uint64_t(1) << 52) | m;
+    uint32_t q = (uint32_t)(S >> sh);
+    const uint64_t rem = S & ((uint64_t(1) << sh) - 1);
+    const uint64_t half = uint64_t(1) << (sh - 1);
+    if (rem > half || (rem == half && (q & 1u))) q += 1u;
+    return __uint_as_float(sign | q);
+}
 
 // Accumulator element -> fp32 gradient (rounded once, to nearest).
 __device__ __forceinline__ float to_f32(float v) { return v; }
-__device__ __forceinline__ float to_f32(double v) { return __double2float_rn(v); }
+__device__ __forceinline__ float to_f32(double v) { return narrow(v); }
+
+// Non-zero test (+0 and -0 are zero), fp64 by its bits.
+__device__ __forceinline__ bool nonzero(float v) { return v != 0.f; }
+__device__ __forceinline__ bool nonzero(double v) {
+    return ((uint64_t)__double_as_longlong(v) << 1) != 0u;
+}
 
 __device__ __forceinline__ bool bag_range(const int64_t* __restrict__ off, int64_t s, int64_t nnz,
                                           int64_t& q0, int64_t& q1) {

@@ -45,7 +45,7 @@ struct Touched {
 struct SortedBuffers {
     uint32_t* pair_x;             // nnz*J buckets written by the forward (0xffffffff: bad id)
     uint32_t* q_row;              // nnz output rows b*T + t written by the forward
-    uint32_t* cnt;                // R per-bucket counts, filled by the forward
+    uint32_t* cnt;                // R per-bucket counts, filled by launch_sorted_count
     uint32_t* start;              // R + 1 bucket starts
     uint32_t* bsum;               // per scan chunk: entries, then their exclusive prefix
     uint32_t* bnz;                // per scan chunk: non-empty buckets
@@ -53,6 +53,9 @@ struct SortedBuffers {
     unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j) in bucket order
 };
 int64_t sorted_scan_blocks(int64_t R);
+// Per-bucket counts of the valid pairs (cnt must be zero on entry).
+cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, int sm_count,
+                                cudaStream_t st);
 // Bucket starts; with `touched`, also the list / bitmap of non-empty buckets.
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
                                cudaStream_t st);
@@ -66,13 +69,12 @@ cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const 
 cudaError_t launch_locations(const DevParams& p, const int64_t* idx, int64_t nnz,
                              const int64_t* off, int64_t B, int64_t* locs, DevError* err,
                              int sm_count, cudaStream_t st);
-// Forward; when pair_x / q_row / cnt are given it also writes every pair's
-// bucket, every id's output row and the per-bucket counts for the sorted
-// backward path (cnt must be zero on entry).
+// Forward; when pair_x / q_row are given it also writes every pair's bucket
+// and every id's output row for the sorted backward path.
 cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
-                           DevError* err, uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt,
-                           int sm_count, cudaStream_t st);
+                           DevError* err, uint32_t* pair_x, uint32_t* q_row, int sm_count,
+                           cudaStream_t st);
 // Backward scatter into an fp32 target (scale applied to grad_out) or into an
 // fp64 accumulator (scale 1).
 cudaError_t launch_scatter(const DevParams& p, const RowLayout& lay, const int64_t* idx,
@@ -99,5 +101,8 @@ cudaError_t launch_update_touched64(bool adagrad, float* w, float* Gacc, double*
 cudaError_t launch_grad_export(double* g, float* out, int64_t M, int sm_count, cudaStream_t st);
 // Clears the bitmap words of the listed starts and resets the list count.
 cudaError_t launch_touched_clear(const Touched& touched, int sm_count, cudaStream_t st);
+// direction 0: fp32 -> fp64 (widen); 1: fp64 -> fp32 (narrow), n values.
+cudaError_t launch_convert(int direction, const void* in, void* out, int64_t n, int sm_count,
+                           cudaStream_t st);
 
 }  // namespace pss

@@ -74,7 +74,7 @@ __device__ __forceinline__ bool load4_nonzero<double>(double* g, int64_t i, floa
     const double2 a = reinterpret_cast<const double2*>(g)[2 * i];
     const double2 b = reinterpret_cast<const double2*>(g)[2 * i + 1];
     gv[0] = to_f32(a.x); gv[1] = to_f32(a.y); gv[2] = to_f32(b.x); gv[3] = to_f32(b.y);
-    return a.x != 0.0 || a.y != 0.0 || b.x != 0.0 || b.y != 0.0;
+    return nonzero(a.x) || nonzero(a.y) || nonzero(b.x) || nonzero(b.y);
 }
 __device__ __forceinline__ void zero4(float* g, int64_t i) {
     reinterpret_cast<float4*>(g)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -115,13 +115,26 @@ k_update_dense(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g
         zero4(g, i);
     }
     for (int64_t e = n4 * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < M; e += stride) {
-        if (g[e] == (GT)0) continue;
+        if (!nonzero(g[e])) continue;
         const float gv = to_f32(g[e]);
         if (gv != 0.f) {
             if (ADA) adagrad_elem(w[e], Ga[e], gv, lr, eps);
             else sgd_elem(w[e], gv, lr);
         }
         g[e] = (GT)0;
+    }
+}
+
+// Conversion check: the integer fp32 <-> fp64 conversions of the accumulation
+// path applied to n values.
+__global__ void __launch_bounds__(kThreads)
+k_convert(int direction, const void* __restrict__ in, void* __restrict__ out, int64_t n) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        if (direction == 0)
+            static_cast<double*>(out)[i] = widen(static_cast<const float*>(in)[i]);
+        else
+            static_cast<float*>(out)[i] = narrow(static_cast<const double*>(in)[i]);
     }
 }
 
@@ -132,7 +145,7 @@ k_grad_export(double* __restrict__ g, float* __restrict__ out, int64_t M) {
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < M; e += stride) {
         const double v = g[e];
         out[e] = to_f32(v);
-        if (v != 0.0) g[e] = 0.0;
+        if (nonzero(v)) g[e] = 0.0;
     }
 }
 
@@ -166,7 +179,7 @@ k_update_touched(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__
             if (!owner) continue;
             const int64_t e = (int64_t)x * G + z;
             const GT raw = g[e];
-            if (raw == (GT)0) continue;
+            if (!nonzero(raw)) continue;
             const float gv = to_f32(raw);
             if (gv != 0.f) {
                 if (ADA) adagrad_elem(w[e], Ga[e], gv, lr, eps);
@@ -255,6 +268,14 @@ cudaError_t launch_update_touched64(bool adagrad, float* w, float* Ga, double* g
 cudaError_t launch_grad_export(double* g, float* out, int64_t M, int sm_count, cudaStream_t st) {
     const int grid = grid_for(k_grad_export, sm_count, (M + kThreads - 1) / kThreads);
     k_grad_export<<<grid, kThreads, 0, st>>>(g, out, M);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_convert(int direction, const void* in, void* out, int64_t n, int sm_count,
+                           cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    const int grid = grid_for(k_convert, sm_count, (n + kThreads - 1) / kThreads);
+    k_convert<<<grid, kThreads, 0, st>>>(direction, in, out, n);
     return cudaGetLastError();
 }
 

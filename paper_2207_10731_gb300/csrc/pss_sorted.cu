@@ -5,14 +5,14 @@
 //   pair_x[p]  bucket x of pair p = q*J + j (block start G*x), or 0xffffffff
 //              for an id outside its table;
 //   q_row[q]   output row b*T + t of the bag that holds id q;
-//   cnt[x]     number of valid pairs with bucket x (the forward zeroes and
-//              fills it while it hashes).
 // Steps (all on the caller's stream):
+//   0. count    cnt[x] = number of valid pairs with bucket x (cnt zeroed by
+//               the caller);
 //   1. scan     start[x] = sum of cnt[y] for y < x (three kernels);
 //               statistics: valid pairs and distinct buckets;
-//   2. scatter  each pair takes slot start[x] + (--cnt[x]) of sorted_e, which
-//               holds (x, r = row*J + j): the bucket and the upstream-gradient
-//               chunk to add;
+//   2. scatter  each pair takes a slot in [start[x], start[x+1]) of sorted_e,
+//               which holds (x, r = row*J + j): the bucket and the
+//               upstream-gradient chunk to add;
 //   3. reduce   the sorted entries are cut into tasks of kPiece consecutive
 //               entries; one group of lanes per task owns 16-byte columns of
 //               the block, adds the chunks of each run of equal x with
@@ -160,69 +160,151 @@ k_scan_apply(const uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __rest
     }
 }
 
-// Slot of every valid pair; cnt counts back down to zero.  Lanes of a warp
-// with the same bucket share one atomic (the leader takes n slots at once);
-// each warp keeps kSU such rounds in flight.
-constexpr int kSU = 4;
+// Counting and slot assignment work on SEGMENTS of kSeg consecutive pairs,
+// one per CTA at a time.  The CTA first merges its segment in a shared-memory
+// hash table (bucket -> number of pairs; each pair's rank among the segment's
+// pairs of its bucket), then touches the global counter of every DISTINCT
+// bucket of the segment once.  Under a skewed (Zipf) id distribution a hot
+// bucket therefore sees one global atomic per segment rather than one per
+// pair, so no long queue of atomics forms on one address.
+constexpr int kSegThreads = 256;
+constexpr int kSegPer = 8;                        // pairs per thread
+constexpr int kSeg = kSegThreads * kSegPer;       // pairs per segment
+constexpr int kSegLog2Slots = 12;
+constexpr int kSegSlots = 1 << kSegLog2Slots;     // hash slots (load factor <= 1/2)
+static_assert(kSegSlots >= 2 * kSeg, "the segment table needs a free slot for every key");
+static_assert(kSeg <= 65536 && kSegSlots <= 65536, "slot and rank are packed in 16 bits each");
+constexpr int kSegFlushU = 4;                     // global atomics in flight per thread
+constexpr uint32_t kEmpty = 0xffffffffu;          // == kBad, which is never inserted
 
-__global__ void __launch_bounds__(kThreads)
-k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
-               int J, int log2J, const uint32_t* __restrict__ start, uint32_t* __restrict__ cnt,
-               unsigned long long* __restrict__ sorted_e) {
-    const int lane = threadIdx.x & 31;
-    const int64_t wstride = (int64_t)gridDim.x * blockDim.x * kSU;
-    for (int64_t p0 = ((int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31)) * kSU; p0 < npairs;
-         p0 += wstride) {
-        uint32_t x[kSU], row[kSU], st0[kSU], old[kSU], jj[kSU];
-        unsigned peers[kSU];
-#pragma unroll
-        for (int u = 0; u < kSU; ++u) {
-            const int64_t p = p0 + u * 32 + lane;
-            x[u] = (p < npairs) ? __ldg(pair_x + p) : kBad;
-        }
-        // loads that do not depend on the slot go first, so they overlap the atomics
-#pragma unroll
-        for (int u = 0; u < kSU; ++u) {
-            const uint32_t pp = (uint32_t)(p0 + u * 32 + lane);   // npairs < 2^32 on this path
-            const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
-            jj[u] = pp - q * (uint32_t)J;
-            row[u] = 0;
-            st0[u] = 0;
-            if (x[u] != kBad) {
-                row[u] = __ldg(q_row + q);
-                st0[u] = __ldg(start + x[u]);
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < kSU; ++u) {
-            peers[u] = __match_any_sync(0xffffffffu, x[u]);
-            old[u] = 0;
-            if (x[u] != kBad && lane == __ffs(peers[u]) - 1)
-                old[u] = atomicSub(cnt + x[u], (uint32_t)__popc(peers[u]));
-        }
-#pragma unroll
-        for (int u = 0; u < kSU; ++u) {
-            const int leader = __ffs(peers[u]) - 1;
-            const uint32_t o = __shfl_sync(0xffffffffu, old[u], leader);
-            if (x[u] == kBad) continue;
-            const uint32_t rank = (uint32_t)__popc(peers[u] & ((1u << lane) - 1u));
-            const uint32_t slot = st0[u] + o - 1u - rank;
-            sorted_e[slot] = ((unsigned long long)x[u] << 32) | (row[u] * (uint32_t)J + jj[u]);
-        }
+// Insert bucket x (not kBad) into the segment table; returns the slot in the
+// low 16 bits and the pair's rank among the segment's pairs of bucket x in
+// the high 16 bits.  Linear probing always ends: the table has more slots
+// than a segment has pairs.
+__device__ __forceinline__ uint32_t seg_insert(uint32_t* s_key, uint32_t* s_val, uint32_t x) {
+    uint32_t h = (x * 0x9e3779b1u) >> (32 - kSegLog2Slots);
+    for (int probe = 0; probe < kSegSlots; ++probe) {
+        const uint32_t prev = atomicCAS(s_key + h, kEmpty, x);
+        if (prev == kEmpty || prev == x) break;
+        h = (h + 1u) & (uint32_t)(kSegSlots - 1);
+    }
+    return h | (atomicAdd(s_val + h, 1u) << 16);
+}
+
+__device__ __forceinline__ void seg_table_init(uint32_t* s_key, uint32_t* s_val) {
+    for (int i = threadIdx.x; i < kSegSlots; i += kSegThreads) {
+        s_key[i] = kEmpty;
+        s_val[i] = 0u;
     }
 }
 
-// Exact fp32 -> fp64 widening from the IEEE-754 fields (integer pipe): the
-// exponent is re-biased (127 -> 1023) and the 23-bit fraction moved to the top
-// of the 52-bit one.  Zeros, subnormals, infinities and NaNs take the
-// hardware conversion.
-__device__ __forceinline__ double widen(float f) {
-    const uint32_t u = __float_as_uint(f);
-    const uint32_t e = (u >> 23) & 0xffu;
-    if (e == 0u || e == 0xffu) return (double)f;
-    const uint64_t bits = ((uint64_t)(u & 0x80000000u) << 32) |
-                          ((uint64_t)(e + 896u) << 52) | ((uint64_t)(u & 0x7fffffu) << 29);
-    return __longlong_as_double((long long)bits);
+// cnt[x] += number of valid pairs with bucket x.
+__global__ void __launch_bounds__(kSegThreads)
+k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t* __restrict__ cnt) {
+    __shared__ uint32_t s_key[kSegSlots];
+    __shared__ uint32_t s_val[kSegSlots];
+    seg_table_init(s_key, s_val);
+    const int64_t nseg = (npairs + kSeg - 1) / kSeg;
+    for (int64_t seg = blockIdx.x; seg < nseg; seg += gridDim.x) {
+        const int64_t p0 = seg * kSeg;
+        uint32_t x[kSegPer], hr[kSegPer];
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i) {
+            const int64_t p = p0 + i * kSegThreads + threadIdx.x;
+            x[i] = (p < npairs) ? __ldg(pair_x + p) : kBad;
+        }
+        __syncthreads();   // the previous segment's table is clear
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i)
+            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i]) : 0u;
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < kSegSlots / kSegThreads; ++k) {
+            const int sl = k * kSegThreads + threadIdx.x;
+            const uint32_t key = s_key[sl];
+            if (key != kEmpty) atomicAdd(cnt + key, s_val[sl]);
+        }
+        __syncthreads();
+        // each thread clears the slots of its own pairs
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i)
+            if (x[i] != kBad) {
+                s_key[hr[i] & 0xffffu] = kEmpty;
+                s_val[hr[i] & 0xffffu] = 0u;
+            }
+    }
+}
+
+// Slot of every valid pair: cnt counts back down to zero, each segment taking
+// one contiguous range of every bucket it holds (one atomic per distinct
+// bucket); within the range a pair's place is its rank in the segment table.
+// sorted_e[slot] = x << 32 | row*J + j.
+__global__ void __launch_bounds__(kSegThreads)
+k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
+               int J, int log2J, const uint32_t* __restrict__ start, uint32_t* __restrict__ cnt,
+               unsigned long long* __restrict__ sorted_e) {
+    __shared__ uint32_t s_key[kSegSlots];
+    __shared__ uint32_t s_val[kSegSlots];
+    seg_table_init(s_key, s_val);
+    const int64_t nseg = (npairs + kSeg - 1) / kSeg;
+    for (int64_t seg = blockIdx.x; seg < nseg; seg += gridDim.x) {
+        const int64_t p0 = seg * kSeg;
+        uint32_t x[kSegPer], hr[kSegPer], e[kSegPer], st0[kSegPer];
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i) {
+            const int64_t p = p0 + i * kSegThreads + threadIdx.x;
+            x[i] = (p < npairs) ? __ldg(pair_x + p) : kBad;
+        }
+        // loads that do not depend on the table go first, so they overlap it
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i) {
+            const uint32_t pp = (uint32_t)(p0 + i * kSegThreads + threadIdx.x);  // npairs < 2^32 here
+            const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
+            e[i] = pp - q * (uint32_t)J;
+            st0[i] = 0u;
+            if (x[i] != kBad) {
+                e[i] += __ldg(q_row + q) * (uint32_t)J;
+                st0[i] = __ldg(start + x[i]);
+            }
+        }
+        __syncthreads();   // the previous segment's table is clear
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i)
+            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i]) : 0u;
+        __syncthreads();
+        // one countdown per distinct bucket, kSegFlushU in flight per thread;
+        // the slot's value becomes the segment's first place in the bucket
+#pragma unroll
+        for (int k0 = 0; k0 < kSegSlots / kSegThreads; k0 += kSegFlushU) {
+            uint32_t key[kSegFlushU], c[kSegFlushU], old[kSegFlushU];
+#pragma unroll
+            for (int u = 0; u < kSegFlushU; ++u) {
+                const int sl = (k0 + u) * kSegThreads + threadIdx.x;
+                key[u] = s_key[sl];
+                c[u] = s_val[sl];
+            }
+#pragma unroll
+            for (int u = 0; u < kSegFlushU; ++u)
+                old[u] = (key[u] != kEmpty) ? atomicSub(cnt + key[u], c[u]) : 0u;
+#pragma unroll
+            for (int u = 0; u < kSegFlushU; ++u)
+                if (key[u] != kEmpty) s_val[(k0 + u) * kSegThreads + threadIdx.x] = old[u] - c[u];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i) {
+            if (x[i] == kBad) continue;
+            const uint32_t slot = st0[i] + s_val[hr[i] & 0xffffu] + (hr[i] >> 16);
+            sorted_e[slot] = ((unsigned long long)x[i] << 32) | e[i];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kSegPer; ++i)
+            if (x[i] != kBad) {
+                s_key[hr[i] & 0xffffu] = kEmpty;
+                s_val[hr[i] & 0xffffu] = 0u;
+            }
+    }
 }
 
 // Reduce: one group of gs lanes per task of kPiece sorted entries; lane lg
@@ -638,9 +720,18 @@ cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
                                   cudaStream_t st) {
     const int log2J = (J & (J - 1)) == 0 ? ceil_log2(J) : -1;
-    const int grid = grid_for(k_sort_scatter, sm_count, (npairs + kThreads - 1) / kThreads);
-    k_sort_scatter<<<grid, kThreads, 0, st>>>(sb.pair_x, npairs, sb.q_row, J, log2J, sb.start,
-                                              sb.cnt, sb.sorted_e);
+    const int64_t nseg = (npairs + kSeg - 1) / kSeg;
+    const int grid = grid_for(k_sort_scatter, sm_count, nseg);
+    k_sort_scatter<<<grid, kSegThreads, 0, st>>>(sb.pair_x, npairs, sb.q_row, J, log2J, sb.start,
+                                                 sb.cnt, sb.sorted_e);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, int sm_count,
+                                cudaStream_t st) {
+    const int64_t nseg = (npairs + kSeg - 1) / kSeg;
+    const int grid = grid_for(k_sort_count, sm_count, nseg);
+    k_sort_count<<<grid, kSegThreads, 0, st>>>(sb.pair_x, npairs, sb.cnt);
     return cudaGetLastError();
 }
 

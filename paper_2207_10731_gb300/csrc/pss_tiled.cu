@@ -102,13 +102,12 @@ __device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t*
 constexpr int kWarpPairs = 512;   // staged pairs per warp and round
 
 // Hash the pairs [0, nq*J) of ids qc0.. into s_x (warp-cooperative); emits
-// buckets / counts for the sorted backward when asked.  Counts of equal
-// buckets within the 32 pairs of a round are merged before the atomic.
+// the buckets for the sorted backward when asked.
 template <typename XT>
 __device__ __forceinline__ void warp_stage(const DevParams& p, const int64_t* __restrict__ idx,
                                            int t, uint64_t card, int64_t qc0, int nq, XT* s_x,
                                            DevError* err, uint32_t* __restrict__ pair_x,
-                                           uint32_t* __restrict__ cnt, int lane) {
+                                           int lane) {
     const int npairs = nq * p.J;
     const bool jpow2 = (p.J & (p.J - 1)) == 0;
     const int log2J = 31 - __clz(p.J);
@@ -125,11 +124,6 @@ __device__ __forceinline__ void warp_stage(const DevParams& p, const int64_t* __
             s_x[k] = x;
             if (pair_x) pair_x[qc0 * p.J + k] = (uint32_t)x;
         }
-        if (cnt) {
-            const unsigned peers = __match_any_sync(0xffffffffu, (uint32_t)x);
-            if (x != Invalid<XT>::v && lane == __ffs(peers) - 1)
-                atomicAdd(cnt + (uint64_t)x, (uint32_t)__popc(peers));
-        }
     }
     __syncwarp();
 }
@@ -142,8 +136,7 @@ __device__ __forceinline__ void warp_stage_bags(const DevParams& p, const int64_
                                                 int t, uint64_t card, const int64_t* s_off, int nb,
                                                 XT* s_x, DevError* err,
                                                 uint32_t* __restrict__ pair_x,
-                                                uint32_t* __restrict__ q_row,
-                                                uint32_t* __restrict__ cnt, uint32_t row0,
+                                                uint32_t* __restrict__ q_row, uint32_t row0,
                                                 int lane) {
     const int npairs = nb * p.J;
     const bool jpow2 = (p.J & (p.J - 1)) == 0;
@@ -164,11 +157,6 @@ __device__ __forceinline__ void warp_stage_bags(const DevParams& p, const int64_
             }
             s_x[k] = x;
         }
-        if (cnt) {
-            const unsigned peers = __match_any_sync(0xffffffffu, (uint32_t)x);
-            if (x != Invalid<XT>::v && lane == __ffs(peers) - 1)
-                atomicAdd(cnt + (uint64_t)x, (uint32_t)__popc(peers));
-        }
     }
     __syncwarp();
 }
@@ -178,7 +166,7 @@ __global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
 k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                const int64_t* __restrict__ off, int64_t B, const float* __restrict__ w,
                float* __restrict__ out, DevError* err, uint32_t* __restrict__ pair_x,
-               uint32_t* __restrict__ q_row, uint32_t* __restrict__ cnt, int log2gs, int wb,
+               uint32_t* __restrict__ q_row, int log2gs, int wb,
                int tiles_per_table) {
     using V = Vec<VW>;
     using VT = typename V::T;
@@ -239,7 +227,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
 
         if (!multi && nb * J <= kWarpPairs) {
             // every bag holds at most one id: one load per bag, no accumulation
-            warp_stage_bags<XT>(p, idx, t, card, s_off, nb, s_x, err, pair_x, q_row, cnt,
+            warp_stage_bags<XT>(p, idx, t, card, s_off, nb, s_x, err, pair_x, q_row,
                                 (uint32_t)(b0 * p.T + t), lane);
             float* orow0 = obase + gb0 * ostride;
             for (int bb0 = gb0; bb0 < gb1; bb0 += kU) {
@@ -289,8 +277,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                 if (q >= sw1) {
                     sw0 = q;
                     sw1 = (qb - q) < qcw ? qb : q + qcw;
-                    warp_stage<XT>(p, idx, t, card, sw0, (int)(sw1 - sw0), s_x, err, pair_x, cnt,
-                                   lane);
+                    warp_stage<XT>(p, idx, t, card, sw0, (int)(sw1 - sw0), s_x, err, pair_x, lane);
                 }
                 const int64_t qend = c < sw1 ? c : sw1;
                 for (int64_t qs = q; qs < qend; qs += (int64_t)kU * ng) {
@@ -466,7 +453,7 @@ size_t tile_smem(const TileGeom& g, const DevParams& p, size_t xbytes) {
 template <int VW, int KC, typename XT>
 cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                      const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
-                     uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt, int sm_count,
+                     uint32_t* pair_x, uint32_t* q_row, int sm_count,
                      cudaStream_t st) {
     const int wb = (32 >> lay.log2gs) * kBagsPerGroup;      // bags per warp tile
     const int tpt = (int)((B + wb - 1) / wb);
@@ -477,7 +464,7 @@ cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* id
     const int grid = grid_for(k_forward_warp<VW, KC, XT>, sm_count, (ntiles + kWarps - 1) / kWarps,
                               smem);
     k_forward_warp<VW, KC, XT><<<grid, kThreads, smem, st>>>(p, idx, nnz, off, B, w, out, err,
-                                                             pair_x, q_row, cnt, lay.log2gs, wb,
+                                                             pair_x, q_row, lay.log2gs, wb,
                                                              tpt);
     return cudaGetLastError();
 }
@@ -498,13 +485,13 @@ cudaError_t sc_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx
 template <int VW, int KC>
 cudaError_t fwd_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                   const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
-                  uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt, int sm_count,
+                  uint32_t* pair_x, uint32_t* q_row, int sm_count,
                   cudaStream_t st) {
     if (p.R < 0xffffffffull)
         return fwd_inst<VW, KC, uint32_t>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row,
-                                          cnt, sm_count, st);
+                                          sm_count, st);
     return fwd_inst<VW, KC, uint64_t>(p, lay, idx, nnz, off, B, w, out, err, nullptr, nullptr,
-                                      nullptr, sm_count, st);
+                                      sm_count, st);
 }
 
 template <int VW, int KC, typename AT>
@@ -531,10 +518,10 @@ cudaError_t sc_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, i
 
 cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
-                           DevError* err, uint32_t* pair_x, uint32_t* q_row, uint32_t* cnt,
-                           int sm_count, cudaStream_t st) {
+                           DevError* err, uint32_t* pair_x, uint32_t* q_row, int sm_count,
+                           cudaStream_t st) {
 #define PSS_FW(VW, KC) \
-    return fwd_x<VW, KC>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row, cnt, sm_count, st)
+    return fwd_x<VW, KC>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row, sm_count, st)
     if (lay.vw == 4) {
         switch (lay.kc) {
             case 1: PSS_FW(4, 1);

@@ -71,3 +71,10 @@ def test_null_handle_calls_are_rejected(lib):
         binding.PSS_ERR_INVALID_ARG
     assert lib.pss_set_option(None, 1, 0) == binding.PSS_ERR_INVALID_ARG
     assert lib.pss_destroy(None) == binding.PSS_OK
+
+
+def test_check_convert_rejects_bad_arguments_before_touching_the_device(lib):
+    for direction, n in ((2, 4), (-1, 4), (0, -1)):
+        rc = lib.pss_check_convert(direction, None, None, n, None)
+        assert rc == binding.PSS_ERR_INVALID_ARG
+    assert lib.pss_check_convert(1, None, None, 0, None) == binding.PSS_OK

@@ -81,6 +81,7 @@ FWD_CASES = [
     dict(name="tiny", Z=1, G=1),
     dict(name="kaggle", Z=3, G=2, B=300),
     dict(name="tb", B=1000, d=200, Z=32),                    # two columns per lane
+    dict(name="tb", B=600, d=384, Z=64, G=8),                # three 16-byte columns per lane
     dict(name="tb", B=500, d=10, Z=4, G=4),                  # d not a multiple of 4
 ]
 
@@ -136,6 +137,28 @@ def test_grad_parity(case, path):
     assert abs(g.astype(np.float64).sum() - mass) <= 1e-5 * A.sum() + 1e-6
     if path != "auto":
         assert h.info()["last_path"] == PATHS[path]
+    h.close()
+
+
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
+def test_grad_single_hot_id_and_repeated_backward(path):
+    # Every bag of every table holds id 0, so each table's J buckets collect
+    # all B contributions (the most skewed batch there is); B is not a
+    # multiple of any segment or tile size.  A second backward of the same
+    # batch must give the same gradient.
+    w = wl.make_workload("tb", B=5003)
+    w.indices[:] = 0
+    h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    h.forward(*_batch_cuda(w), w.B)
+    go = gu.cuda(w.grad_out)
+    g1 = gu.host(h.backward_grad(go))
+    g2 = gu.host(h.backward_grad(go))
+    ref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
+    A = o.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g1, ref, A)
+    gu.check_grad(g2, ref, A)
+    assert h.info()["last_path"] == PATHS[path]
     h.close()
 
 
@@ -262,6 +285,7 @@ def test_sorted_path_reports_collision_rate():
     info = h.info()
     locs, _ = o.locations(w.indices, w.offsets, w.B)
     want = 1.0 - np.unique(locs).shape[0] / locs.shape[0]
+    assert 0.0 < want < 1.0
     assert info["last_path"] == binding.PATH_SORTED
     assert abs(info["last_collision_rate"] - want) < 1e-12
     h.close()
@@ -519,6 +543,6 @@ def test_profile_and_launch_counts():
     h.forward(idx, off, w.B)
     h.backward_update(go, w.lr)
     assert h.profile(binding.K_SORT)[0] == 1 and h.profile(binding.K_REDUCE)[0] == 1
-    # forward (which also counts buckets), 3 scan kernels, scatter, reduce, update
-    assert h.info()["kernel_launches"] - before == 7
+    # forward, bucket count, 3 scan kernels, slot scatter, reduce, update
+    assert h.info()["kernel_launches"] - before == 8
     h.close()
