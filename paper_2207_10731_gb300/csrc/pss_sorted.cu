@@ -31,7 +31,7 @@ namespace {
 
 constexpr uint32_t kBad = 0xffffffffu;
 constexpr int kScanThreads = 1024;
-constexpr int kScanPerThread = 8;
+constexpr int kScanPerThread = 2;
 constexpr int kScanChunk = kScanThreads * kScanPerThread;
 constexpr int kRU = 4;            // entries in flight per group (summed as a tree when they
                                   // all continue the current run)
@@ -599,7 +599,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                     const int part = pc & 7;
                     const int e = st * kAS + i;
                     if (e < n) {
-                        const uint32_t r = (uint32_t)ent[e];
+                        const uint32_t r = reinterpret_cast<const uint32_t*>(ent)[2 * e];  // low word
                         cp_async16(&s_ring[warp][st % kAD][i][part * 4],
                                    gout + (uint64_t)r * 32u + (uint32_t)(part * 4));
                     }
@@ -616,19 +616,24 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
             cp_async_wait<kAD - 1>();
             __syncwarp();
             const float* buf = &s_ring[warp][st % kAD][0][0];
-            uint32_t xs[kAS];
+            const uint32_t* ex = reinterpret_cast<const uint32_t*>(ent + st * kAS) + 1;  // high words: x
+            // the entries are sorted and padded with kBad: when the stage's last
+            // bucket continues the run, the stage is full and all of it does
+            // all loads first, in one round trip (the flush's reduction is a
+            // memory barrier for the compiler, so later loads would not overlap);
+            // chunks past the task's end are never read as values
+            const uint32_t xlast = ex[2 * (kAS - 1)];
             float v[kAS];
 #pragma unroll
-            for (int i = 0; i < kAS; ++i) {
-                const int e = st * kAS + i;
-                xs[i] = (e < n) ? (uint32_t)(ent[e] >> 32) : kBad;
-                v[i] = (e < n) ? buf[i * 32 + lane] : 0.f;
-            }
-            if (xs[kAS - 1] == cur) {
+            for (int i = 0; i < kAS; ++i) v[i] = buf[i * 32 + lane];
+            if (xlast == cur) {
                 const float a = (v[0] + v[1]) + (v[2] + v[3]);
                 const float b = (v[4] + v[5]) + (v[6] + v[7]);
                 kahan_add(sum, comp, a + b);
             } else {
+                uint32_t xs[kAS];
+#pragma unroll
+                for (int i = 0; i < kAS; ++i) xs[i] = ex[2 * i];
 #pragma unroll
                 for (int i = 0; i < kAS; ++i) {
                     if (xs[i] == kBad) break;
