@@ -594,7 +594,8 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool touch, c
     const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
     if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
     poll_stats(h);
-    PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)h->dp.R, st));
+    // cnt is zero here: it is zeroed when allocated, and every sort's slot
+    // scatter counts each bucket back down by exactly what its count added
     {
         LaunchScope ls(h, PSS_K_SORT, st, 5);
         PSS_TRY(launch_sorted_count(h->sb, npairs, h->sm_count, st));

@@ -64,6 +64,33 @@ __device__ __forceinline__ void kahan_add(float& s, float& c, float x) {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 
+// Programmatic dependent launch.  Every kernel of the library starts with
+// pdl_prologue(), which waits until the previous kernel on the stream has
+// completed and its memory is visible (a no-op when the previous work was not
+// a kernel launched this way), before any global access.  So a kernel never
+// overlaps the one before it in anything it reads or writes; only the launch
+// latency between them is hidden.
+__device__ __forceinline__ void pdl_prologue() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Launch with programmatic stream serialization (see pdl_prologue).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                     cudaStream_t st, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 inline int ceil_log2(int v) {
     int l = 0;
     while ((1 << l) < v) ++l;

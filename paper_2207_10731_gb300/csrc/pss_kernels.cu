@@ -24,6 +24,7 @@ __global__ void __launch_bounds__(kThreads)
 k_locations(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
             const int64_t* __restrict__ off, int64_t B, uint64_t Binv, int64_t* __restrict__ locs,
             DevError* err) {
+    pdl_prologue();
     const int64_t nbags = (int64_t)p.T * B;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; s < nbags; s += stride) {
@@ -90,6 +91,7 @@ template <bool ADA, typename GT>
 __global__ void __launch_bounds__(kThreads)
 k_update_dense(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g, int64_t M,
                float lr, float eps) {
+    pdl_prologue();
     const int64_t n4 = M >> 2;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     float4* w4 = reinterpret_cast<float4*>(w);
@@ -129,6 +131,7 @@ k_update_dense(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g
 // path applied to n values.
 __global__ void __launch_bounds__(kThreads)
 k_convert(int direction, const void* __restrict__ in, void* __restrict__ out, int64_t n) {
+    pdl_prologue();
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
         if (direction == 0)
@@ -141,6 +144,7 @@ k_convert(int direction, const void* __restrict__ in, void* __restrict__ out, in
 // Gradient export: out[e] = fp32(g[e]) and g[e] = 0, over all of M.
 __global__ void __launch_bounds__(kThreads)
 k_grad_export(double* __restrict__ g, float* __restrict__ out, int64_t M) {
+    pdl_prologue();
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < M; e += stride) {
         const double v = g[e];
@@ -157,6 +161,7 @@ template <bool ADA, typename GT>
 __global__ void __launch_bounds__(kThreads)
 k_update_touched(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g,
                  Touched tc, int64_t G, int L, float lr, float eps) {
+    pdl_prologue();
     const int lane = threadIdx.x & 31;
     unsigned long long n = *tc.count;
     if ((int64_t)n > tc.cap) n = (unsigned long long)tc.cap;
@@ -191,6 +196,7 @@ k_update_touched(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__
 }
 
 __global__ void __launch_bounds__(kThreads) k_touched_clear(Touched tc) {
+    pdl_prologue();
     unsigned long long n = *tc.count;
     if ((int64_t)n > tc.cap) n = (unsigned long long)tc.cap;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -202,16 +208,16 @@ template <bool ADA, typename GT>
 cudaError_t update_dense_inst(float* w, float* Ga, GT* g, int64_t M, float lr, float eps,
                               int sm_count, cudaStream_t st) {
     const int grid = grid_for(k_update_dense<ADA, GT>, sm_count, ((M >> 2) + kThreads) / kThreads);
-    k_update_dense<ADA, GT><<<grid, kThreads, 0, st>>>(w, Ga, g, M, lr, eps);
-    return cudaGetLastError();
+    return launch_k(k_update_dense<ADA, GT>, dim3(grid), dim3(kThreads), 0, st, w, Ga, g, M, lr,
+                    eps);
 }
 
 template <bool ADA, typename GT>
 cudaError_t update_touched_inst(float* w, float* Ga, GT* g, const Touched& tc, int64_t G,
                                 int32_t L, float lr, float eps, int sm_count, cudaStream_t st) {
     const int grid = grid_for(k_update_touched<ADA, GT>, sm_count, (tc.cap + kWarps - 1) / kWarps);
-    k_update_touched<ADA, GT><<<grid, kThreads, 0, st>>>(w, Ga, g, tc, G, L, lr, eps);
-    return cudaGetLastError();
+    return launch_k(k_update_touched<ADA, GT>, dim3(grid), dim3(kThreads), 0, st, w, Ga, g, tc, G,
+                    L, lr, eps);
 }
 
 }  // namespace
@@ -235,8 +241,8 @@ cudaError_t launch_locations(const DevParams& p, const int64_t* idx, int64_t nnz
                              int sm_count, cudaStream_t st) {
     const int64_t nbags = (int64_t)p.T * B;
     const int grid = grid_for(k_locations, sm_count, (nbags + kThreads - 1) / kThreads);
-    k_locations<<<grid, kThreads, 0, st>>>(p, idx, nnz, off, B, UINT64_MAX / (uint64_t)B, locs, err);
-    return cudaGetLastError();
+    return launch_k(k_locations, dim3(grid), dim3(kThreads), 0, st, p, idx, nnz, off, B,
+                    UINT64_MAX / (uint64_t)B, locs, err);
 }
 
 cudaError_t launch_update_dense(bool adagrad, float* w, float* Ga, float* g, int64_t M, float lr,
@@ -267,22 +273,19 @@ cudaError_t launch_update_touched64(bool adagrad, float* w, float* Ga, double* g
 
 cudaError_t launch_grad_export(double* g, float* out, int64_t M, int sm_count, cudaStream_t st) {
     const int grid = grid_for(k_grad_export, sm_count, (M + kThreads - 1) / kThreads);
-    k_grad_export<<<grid, kThreads, 0, st>>>(g, out, M);
-    return cudaGetLastError();
+    return launch_k(k_grad_export, dim3(grid), dim3(kThreads), 0, st, g, out, M);
 }
 
 cudaError_t launch_convert(int direction, const void* in, void* out, int64_t n, int sm_count,
                            cudaStream_t st) {
     if (n <= 0) return cudaSuccess;
     const int grid = grid_for(k_convert, sm_count, (n + kThreads - 1) / kThreads);
-    k_convert<<<grid, kThreads, 0, st>>>(direction, in, out, n);
-    return cudaGetLastError();
+    return launch_k(k_convert, dim3(grid), dim3(kThreads), 0, st, direction, in, out, n);
 }
 
 cudaError_t launch_touched_clear(const Touched& tc, int sm_count, cudaStream_t st) {
     const int grid = grid_for(k_touched_clear, sm_count, (tc.cap + kThreads - 1) / kThreads);
-    k_touched_clear<<<grid, kThreads, 0, st>>>(tc);
-    cudaError_t e = cudaGetLastError();
+    const cudaError_t e = launch_k(k_touched_clear, dim3(grid), dim3(kThreads), 0, st, tc);
     if (e != cudaSuccess) return e;
     return cudaMemsetAsync(tc.count, 0, sizeof(unsigned long long), st);
 }

@@ -12,6 +12,7 @@
 #include <mutex>
 
 #include "pss.h"
+#include "pss_device.cuh"
 #include "pss_internal.h"
 
 using namespace pss;
@@ -87,6 +88,7 @@ void params_from_seed(uint64_t seed, uint64_t* A, uint64_t* B0) {
 }
 
 __global__ void k_error_report(const DevError* err, int64_t* first_bad) {
+    pdl_prologue();
     if (threadIdx.x == 0 && blockIdx.x == 0) {
         int64_t v = (err->first_bad == ULLONG_MAX) ? -1 : (int64_t)err->first_bad;
         if (v < 0 && (err->flags & kErrOffsets)) v = -2;
@@ -164,8 +166,8 @@ extern "C" pss_status pss_grad_noalloc(const int64_t* cards, int32_t T, int32_t 
     }
     if (launch_grad_export(sym.accum, grad, M, sms, st) != cudaSuccess) return PSS_ERR_CUDA;
     if (first_bad) {
-        k_error_report<<<1, 32, 0, st>>>(sym.err, first_bad);
-        if (cudaGetLastError() != cudaSuccess) return PSS_ERR_CUDA;
+        if (launch_k(k_error_report, dim3(1), dim3(32), 0, st, sym.err, first_bad) != cudaSuccess)
+            return PSS_ERR_CUDA;
     }
     return PSS_OK;
 }

@@ -71,6 +71,7 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict__ bsum,
               uint32_t* __restrict__ bnz) {
+    pdl_prologue();
     __shared__ uint32_t s_warp[33];
     const int64_t base = (int64_t)blockIdx.x * kScanChunk;
     uint32_t sum = 0, nz = 0;
@@ -96,6 +97,7 @@ k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict_
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ bnz, int64_t nblk,
            unsigned long long* __restrict__ stats, unsigned long long* __restrict__ touched_count) {
+    pdl_prologue();
     __shared__ uint32_t s_warp[33];
     __shared__ uint32_t s_carry[2];
     if (threadIdx.x < 2) s_carry[threadIdx.x] = 0;
@@ -132,6 +134,7 @@ k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ bnz, int64_t nblk
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_apply(const uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __restrict__ bsum,
              const uint32_t* __restrict__ bnz, uint32_t* __restrict__ start, Touched tc) {
+    pdl_prologue();
     __shared__ uint32_t s_warp[33];
     const int64_t base = (int64_t)blockIdx.x * kScanChunk;
     uint32_t c[kScanPerThread];
@@ -201,6 +204,7 @@ __device__ __forceinline__ void seg_table_init(uint32_t* s_key, uint32_t* s_val)
 // cnt[x] += number of valid pairs with bucket x.
 __global__ void __launch_bounds__(kSegThreads)
 k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t* __restrict__ cnt) {
+    pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
     __shared__ uint32_t s_val[kSegSlots];
     seg_table_init(s_key, s_val);
@@ -243,6 +247,7 @@ __global__ void __launch_bounds__(kSegThreads)
 k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
                int J, int log2J, const uint32_t* __restrict__ start, uint32_t* __restrict__ cnt,
                unsigned long long* __restrict__ sorted_e) {
+    pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
     __shared__ uint32_t s_val[kSegSlots];
     seg_table_init(s_key, s_val);
@@ -320,6 +325,7 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                const unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
                double* __restrict__ g, int log2gs) {
+    pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
     extern __shared__ __align__(16) float s_stage[];   // [groups per CTA][L]
@@ -462,6 +468,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     const unsigned long long* __restrict__ stats, int64_t npairs,
                     const float* __restrict__ gout, int d, int Z, int J, int log2J, int L,
                     int64_t G, double* __restrict__ g) {
+    pdl_prologue();
     __shared__ unsigned long long s_ent[kWarps][kPiece];
     const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
     const int64_t ntasks = (total + kPiece - 1) / kPiece;
@@ -567,6 +574,7 @@ __global__ void __launch_bounds__(kThreads)
 k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                const unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int64_t G, double* __restrict__ g) {
+    pdl_prologue();
     __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
     __shared__ unsigned long long s_ent[kWarps][kAPiece];
     const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
@@ -659,9 +667,8 @@ cudaError_t warp_reduce_launch(const SortedBuffers& sb, int64_t npairs, const fl
     const int64_t ntasks = (npairs + kPiece - 1) / kPiece;   // upper bound
     const int grid = grid_for(k_warp_range_reduce<KE, ZDIV, JPOW2>, sm_count,
                               (ntasks + kWarps - 1) / kWarps);
-    k_warp_range_reduce<KE, ZDIV, JPOW2><<<grid, kThreads, 0, st>>>(
-        sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g);
-    return cudaGetLastError();
+    return launch_k(k_warp_range_reduce<KE, ZDIV, JPOW2>, dim3(grid), dim3(kThreads), 0, st,
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g);
 }
 
 template <int KE>
@@ -684,9 +691,8 @@ cudaError_t reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* 
     const int64_t ntasks = (npairs + kPiece - 1) / kPiece;   // upper bound
     const int64_t work_blocks = (ntasks + gpc - 1) / gpc;
     const int grid = grid_for(k_range_reduce<VW, KC, JPOW2, ZDIV>, sm_count, work_blocks, smem);
-    k_range_reduce<VW, KC, JPOW2, ZDIV><<<grid, kThreads, smem, st>>>(
-        sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, log2gs);
-    return cudaGetLastError();
+    return launch_k(k_range_reduce<VW, KC, JPOW2, ZDIV>, dim3(grid), dim3(kThreads), smem, st,
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, log2gs);
 }
 
 template <int VW, int KC>
@@ -712,14 +718,14 @@ cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched
                                cudaStream_t st) {
     const int64_t nblk = sorted_scan_blocks(R);
     const Touched tc = touched ? *touched : Touched{};
-    k_scan_reduce<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.bnz);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_k(k_scan_reduce, dim3((unsigned)nblk), dim3(kScanThreads), 0, st,
+                             sb.cnt, R, sb.bsum, sb.bnz);
     if (e != cudaSuccess) return e;
-    k_scan_top<<<1, kScanThreads, 0, st>>>(sb.bsum, sb.bnz, nblk, sb.stats, tc.count);
-    e = cudaGetLastError();
+    e = launch_k(k_scan_top, dim3(1), dim3(kScanThreads), 0, st, sb.bsum, sb.bnz, nblk, sb.stats,
+                 tc.count);
     if (e != cudaSuccess) return e;
-    k_scan_apply<<<(unsigned)nblk, kScanThreads, 0, st>>>(sb.cnt, R, sb.bsum, sb.bnz, sb.start, tc);
-    return cudaGetLastError();
+    return launch_k(k_scan_apply, dim3((unsigned)nblk), dim3(kScanThreads), 0, st, sb.cnt, R,
+                    sb.bsum, sb.bnz, sb.start, tc);
 }
 
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
@@ -727,17 +733,15 @@ cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J
     const int log2J = (J & (J - 1)) == 0 ? ceil_log2(J) : -1;
     const int64_t nseg = (npairs + kSeg - 1) / kSeg;
     const int grid = grid_for(k_sort_scatter, sm_count, nseg);
-    k_sort_scatter<<<grid, kSegThreads, 0, st>>>(sb.pair_x, npairs, sb.q_row, J, log2J, sb.start,
-                                                 sb.cnt, sb.sorted_e);
-    return cudaGetLastError();
+    return launch_k(k_sort_scatter, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs,
+                    sb.q_row, J, log2J, sb.start, sb.cnt, sb.sorted_e);
 }
 
 cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, int sm_count,
                                 cudaStream_t st) {
     const int64_t nseg = (npairs + kSeg - 1) / kSeg;
     const int grid = grid_for(k_sort_count, sm_count, nseg);
-    k_sort_count<<<grid, kSegThreads, 0, st>>>(sb.pair_x, npairs, sb.cnt);
-    return cudaGetLastError();
+    return launch_k(k_sort_count, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs, sb.cnt);
 }
 
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
@@ -746,8 +750,8 @@ cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const 
     if (p.Z == 32 && p.d % 32 == 0 && (((uintptr_t)gout & 15u) == 0)) {
         const int64_t ntasks = (npairs + kAPiece - 1) / kAPiece;   // upper bound
         const int grid = grid_for(k_async_reduce, sm_count, (ntasks + kWarps - 1) / kWarps);
-        k_async_reduce<<<grid, kThreads, 0, st>>>(sb.sorted_e, sb.stats, npairs, gout, p.G, g);
-        return cudaGetLastError();
+        return launch_k(k_async_reduce, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e, sb.stats,
+                        npairs, gout, p.G, g);
     }
     // blocks of 32+ elements: one warp per task, one element per lane
     if (p.L >= 32) {

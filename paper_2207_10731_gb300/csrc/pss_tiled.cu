@@ -168,6 +168,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                float* __restrict__ out, DevError* err, uint32_t* __restrict__ pair_x,
                uint32_t* __restrict__ q_row, int log2gs, int wb,
                int tiles_per_table) {
+    pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
     extern __shared__ __align__(16) unsigned char smem[];
@@ -342,6 +343,7 @@ k_scatter_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                 const int64_t* __restrict__ off, int64_t B, const float* __restrict__ gout,
                 float scale, AT* __restrict__ target, Touched tc, DevError* err, int log2gs,
                 TileGeom tg) {
+    pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
     extern __shared__ __align__(16) unsigned char smem[];
@@ -463,10 +465,8 @@ cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* id
     if (ntiles >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
     const int grid = grid_for(k_forward_warp<VW, KC, XT>, sm_count, (ntiles + kWarps - 1) / kWarps,
                               smem);
-    k_forward_warp<VW, KC, XT><<<grid, kThreads, smem, st>>>(p, idx, nnz, off, B, w, out, err,
-                                                             pair_x, q_row, lay.log2gs, wb,
-                                                             tpt);
-    return cudaGetLastError();
+    return launch_k(k_forward_warp<VW, KC, XT>, dim3(grid), dim3(kThreads), smem, st, p, idx, nnz,
+                    off, B, w, out, err, pair_x, q_row, lay.log2gs, wb, tpt);
 }
 
 template <int VW, int KC, typename XT, typename AT, bool TOUCH>
@@ -477,9 +477,8 @@ cudaError_t sc_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx
     const size_t smem = tile_smem(tg, p, sizeof(XT));
     const int64_t ntiles = (int64_t)p.T * tg.tiles_per_table;
     const int grid = grid_for(k_scatter_tiled<VW, KC, XT, AT, TOUCH>, sm_count, ntiles, smem);
-    k_scatter_tiled<VW, KC, XT, AT, TOUCH><<<grid, kThreads, smem, st>>>(
-        p, idx, nnz, off, B, gout, scale, target, tc, err, lay.log2gs, tg);
-    return cudaGetLastError();
+    return launch_k(k_scatter_tiled<VW, KC, XT, AT, TOUCH>, dim3(grid), dim3(kThreads), smem, st, p,
+                    idx, nnz, off, B, gout, scale, target, tc, err, lay.log2gs, tg);
 }
 
 template <int VW, int KC>
