@@ -38,8 +38,14 @@
  *   `stream` are asynchronous on it (stream-ordered) unless stated otherwise;
  *   the caller's buffers must stay valid until that work completes.  Batch
  *   pointers may be device memory or host memory (pinned or pageable): host
- *   batches are staged through library-owned device buffers on the same
- *   stream.  A handle is not thread-safe; use one handle per thread or lock.
+ *   batches are staged through library-owned device buffers.  Indices,
+ *   offsets and the pooled output move on the call's stream; a host upstream
+ *   gradient is copied on a stream of the library's own, so that the copy
+ *   overlaps the forward and the output's download, and the call's stream
+ *   waits for it before the first kernel that reads it.  Either way, once the
+ *   call's stream has reached the end of the call's work, the library is done
+ *   with the caller's buffers.  A handle is not thread-safe; use one handle
+ *   per thread or lock.
  *
  * Errors: every call returns a pss_status; none aborts the process.  Bad
  * arguments are rejected on the host before any work is queued.  An id outside

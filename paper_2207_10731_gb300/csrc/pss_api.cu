@@ -80,6 +80,14 @@ struct pss_handle {
     bool batch_emitted = false;                 // the last forward wrote pair_x / q_row
     unsigned long long* stats_host = nullptr;   // pinned mirror of sb.stats
     cudaEvent_t stats_ev = nullptr;
+    // a host upstream gradient is copied in on s_h2d, which does not wait for
+    // the caller's stream, so the copy overlaps the forward and the pooled
+    // output's download; the caller's stream waits for ev_grad_ready just
+    // before the first kernel that reads the gradient, and the next copy into
+    // the staging buffer waits for ev_grad_free (its last reader)
+    cudaStream_t s_h2d = nullptr;
+    cudaEvent_t ev_grad_ready = nullptr, ev_grad_free = nullptr, ev_alloc = nullptr;
+    bool grad_free_pending = false;
     bool stats_pending = false;
 
     // profiling
@@ -136,6 +144,58 @@ pss_status device_view(const T* p, size_t count, Staging& s, cudaStream_t st, co
     PSS_TRY(ensure(s, count * sizeof(T), st));
     PSS_TRY(cudaMemcpyAsync(s.ptr, p, count * sizeof(T), cudaMemcpyHostToDevice, st));
     *out = static_cast<const T*>(s.ptr);
+    return PSS_OK;
+}
+
+pss_status ensure_copy_stream(pss_handle* h) {
+    if (h->s_h2d) return PSS_OK;
+    PSS_TRY(cudaStreamCreateWithFlags(&h->s_h2d, cudaStreamNonBlocking));
+    for (cudaEvent_t* e : {&h->ev_grad_ready, &h->ev_grad_free, &h->ev_alloc})
+        PSS_TRY(cudaEventCreateWithFlags(e, cudaEventDisableTiming));
+    return PSS_OK;
+}
+
+// Device view of the upstream gradient.  A host buffer is copied into the
+// staging buffer on s_h2d; *staged tells the caller to call grad_wait before
+// the first kernel that reads it and grad_release after the last one.
+pss_status stage_grad(pss_handle* h, const float* p, size_t count, cudaStream_t st,
+                      const float** out, bool* staged) {
+    *staged = false;
+    if (count == 0 || is_device_ptr(p)) {
+        *out = p;
+        return PSS_OK;
+    }
+    pss_status rc = ensure_copy_stream(h);
+    if (rc != PSS_OK) return rc;
+    const size_t bytes = count * sizeof(float);
+    if (h->st_grad.cap < bytes) {
+        // (re)allocated in the caller's stream order; the copy waits for it
+        PSS_TRY(ensure(h->st_grad, bytes, st));
+        PSS_TRY(cudaEventRecord(h->ev_alloc, st));
+        PSS_TRY(cudaStreamWaitEvent(h->s_h2d, h->ev_alloc, 0));
+    }
+    if (h->grad_free_pending) PSS_TRY(cudaStreamWaitEvent(h->s_h2d, h->ev_grad_free, 0));
+    PSS_TRY(cudaMemcpyAsync(h->st_grad.ptr, p, bytes, cudaMemcpyHostToDevice, h->s_h2d));
+    PSS_TRY(cudaEventRecord(h->ev_grad_ready, h->s_h2d));
+    *out = static_cast<const float*>(h->st_grad.ptr);
+    *staged = true;
+    return PSS_OK;
+}
+
+pss_status grad_wait(pss_handle* h, bool staged, cudaStream_t st) {
+    if (staged) PSS_TRY(cudaStreamWaitEvent(st, h->ev_grad_ready, 0));
+    return PSS_OK;
+}
+
+// After the last reader of a staged gradient.  The caller's stream also waits
+// for the copy here (again, if a reader already did), so that no path returns
+// with the caller's host buffer still being read.
+pss_status grad_release(pss_handle* h, bool staged, cudaStream_t st) {
+    if (staged) {
+        PSS_TRY(cudaStreamWaitEvent(st, h->ev_grad_ready, 0));
+        PSS_TRY(cudaEventRecord(h->ev_grad_free, st));
+        h->grad_free_pending = true;
+    }
     return PSS_OK;
 }
 
@@ -445,6 +505,9 @@ pss_status pss_destroy(pss_handle* h) {
         if (b) cudaFree(b);
     if (h->stats_host) cudaFreeHost(h->stats_host);
     if (h->stats_ev) cudaEventDestroy(h->stats_ev);
+    for (cudaEvent_t e : {h->ev_grad_ready, h->ev_grad_free, h->ev_alloc})
+        if (e) cudaEventDestroy(e);
+    if (h->s_h2d) cudaStreamDestroy(h->s_h2d);
     for (Staging* s : {&h->st_idx, &h->st_off, &h->st_out, &h->st_grad, &h->st_locs})
         if (s->ptr) cudaFree(s->ptr);
     for (int k = 0; k < PSS_K_COUNT; ++k)
@@ -590,7 +653,8 @@ static pss_status scatter_into(pss_handle* h, const float* dgrad, float scale, f
 }
 
 // Sorted path: histogram, scan, scatter by bucket, segmented reduce into g64.
-static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool touch, cudaStream_t st) {
+static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, bool touch,
+                                cudaStream_t st) {
     const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
     if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
     poll_stats(h);
@@ -608,6 +672,10 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool touch, c
         PSS_TRY(cudaEventRecord(h->stats_ev, st));
         h->stats_pending = true;
     }
+    // the sort above needs only the forward's buckets: a host gradient's copy
+    // has overlapped it, and is waited for here
+    pss_status rc = grad_wait(h, staged, st);
+    if (rc != PSS_OK) return rc;
     LaunchScope ls(h, PSS_K_REDUCE, st);
     PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64, h->sm_count, st));
     return PSS_OK;
@@ -621,7 +689,8 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
     DeviceGuard g(h->device);
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const float* dg = nullptr;
-    pss_status rc = device_view(grad_out, (size_t)nbags * (size_t)h->dp.d, h->st_grad, st, &dg);
+    bool staged = false;
+    pss_status rc = stage_grad(h, grad_out, (size_t)nbags * (size_t)h->dp.d, st, &dg, &staged);
     if (rc != PSS_OK) return rc;
     const int64_t pairs = h->last_nnz * (int64_t)h->dp.J;
     const bool ada = h->opt == PSS_ADAGRAD;
@@ -635,7 +704,8 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
         if (rc != PSS_OK) return rc;
         const bool touch = use_touched(h, pairs);
         if (touch && (rc = ensure_touched(h, pairs, st)) != PSS_OK) return rc;
-        if ((rc = sorted_into64(h, dg, touch, st)) != PSS_OK) return rc;
+        if ((rc = sorted_into64(h, dg, staged, touch, st)) != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
         {
             LaunchScope ls(h, PSS_K_UPDATE, st);
             if (touch)
@@ -651,16 +721,20 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
         }
     } else if (h->accum == PSS_ACCUM_F32 && !ada) {
         // SGD is linear in g: scatter -lr * grad_out straight into M.
+        if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
         if (lr != 0.f && (rc = scatter_into(h, dg, -lr, h->w, false, st)) != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
     } else {
         if ((rc = ensure_grad(h, st)) != PSS_OK) return rc;
         const bool touch = use_touched(h, pairs);
         if (touch && (rc = ensure_touched(h, pairs, st)) != PSS_OK) return rc;
+        if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
         if (h->accum == PSS_ACCUM_F32)
             rc = scatter_into(h, dg, 1.0f, h->g, touch, st);
         else
             rc = scatter_into64(h, dg, touch, st);
         if (rc != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
         {
             LaunchScope ls(h, PSS_K_UPDATE, st);
             if (h->accum == PSS_ACCUM_F32) {
@@ -697,7 +771,8 @@ pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, 
     DeviceGuard g(h->device);
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const float* dg = nullptr;
-    pss_status rc = device_view(grad_out, (size_t)nbags * (size_t)h->dp.d, h->st_grad, st, &dg);
+    bool staged = false;
+    pss_status rc = stage_grad(h, grad_out, (size_t)nbags * (size_t)h->dp.d, st, &dg, &staged);
     if (rc != PSS_OK) return rc;
     const bool sorted = h->batch_emitted && want_sorted(h);
     h->last_path = sorted ? PSS_PATH_SORTED : PSS_PATH_ATOMIC;
@@ -707,15 +782,20 @@ pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, 
         rc = ensure_grad(h, st);
         h->accum = saved;
         if (rc != PSS_OK) return rc;
-        if ((rc = sorted_into64(h, dg, false, st)) != PSS_OK) return rc;
+        if ((rc = sorted_into64(h, dg, staged, false, st)) != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
         LaunchScope ls(h, PSS_K_MISC, st);
         PSS_TRY(launch_grad_export(h->g64, grad, h->dp.M, h->sm_count, st));
     } else if (h->accum == PSS_ACCUM_F32) {
         PSS_TRY(cudaMemsetAsync(grad, 0, sizeof(float) * (size_t)h->dp.M, st));
+        if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
         if ((rc = scatter_into(h, dg, 1.0f, grad, false, st)) != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
     } else {
         if ((rc = ensure_grad(h, st)) != PSS_OK) return rc;
+        if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
         if ((rc = scatter_into64(h, dg, false, st)) != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
         LaunchScope ls(h, PSS_K_MISC, st);
         PSS_TRY(launch_grad_export(h->g64, grad, h->dp.M, h->sm_count, st));
     }

@@ -452,6 +452,48 @@ def test_host_buffers_match_device_buffers():
     h2.close()
 
 
+@pytest.mark.parametrize("path", ["sorted", "atomic", "atomic-f32"])
+def test_host_gradient_upload_is_ordered(path):
+    # A host upstream gradient is copied in on the library's own copy stream
+    # (overlapping the forward and the output download).  Three steps through
+    # host buffers, with the pinned gradient buffer overwritten right after
+    # each step's stream synchronisation, must match device buffers bit for
+    # bit (dyadic inputs: every sum is exact on every path).
+    t = gu.torch()
+    w = wl.make_workload("kaggle", grad="dyadic", w0="dyadic")
+    w.lr = 0.125
+    h1, _ = gu.make_pair(w, opt="sgd")
+    h2, _ = gu.make_pair(w, opt="sgd")
+    for h in (h1, h2):
+        h.set_option(binding.OPT_BACKWARD_PATH,
+                     binding.PATH_SORTED if path == "sorted" else binding.PATH_ATOMIC)
+        if path == "atomic-f32":
+            h.set_option(binding.OPT_ACCUM, binding.ACCUM_F32)
+    g_host = t.empty(w.grad_out.shape, dtype=t.float32).pin_memory()
+    out_h = t.empty((w.B, w.T, w.d), dtype=t.float32).pin_memory()
+    for k in range(3):
+        wk = wl.make_workload("kaggle", grad="dyadic", w0="dyadic", batch=k)
+        h1.forward(*_batch_cuda(wk), wk.B)
+        h1.backward_update(gu.cuda(wk.grad_out), w.lr)
+        h2.forward(t.from_numpy(wk.indices).pin_memory(), t.from_numpy(wk.offsets).pin_memory(),
+                   wk.B, out=out_h)
+        g_host.copy_(t.from_numpy(wk.grad_out))
+        h2.backward_update(g_host, w.lr)
+        t.cuda.synchronize()
+        g_host.fill_(float("nan"))
+    np.testing.assert_array_equal(gu.host(h2.get_weights()), gu.host(h1.get_weights()))
+    # a batch whose bags are all empty, with a host gradient: nothing changes
+    before = gu.host(h2.get_weights())
+    empty_off = np.zeros(w.T * w.B + 1, dtype=np.int64)
+    h2.forward(t.from_numpy(np.zeros(0, dtype=np.int64)), t.from_numpy(empty_off), w.B, out=out_h)
+    g_host.copy_(t.from_numpy(w.grad_out))
+    h2.backward_update(g_host, w.lr)
+    t.cuda.synchronize()
+    np.testing.assert_array_equal(gu.host(h2.get_weights()), before)
+    h1.close()
+    h2.close()
+
+
 # --------------------------------------------------------------------------
 # errors: reported, never a trap
 @pytest.mark.parametrize("path", ["atomic", "sorted"])
