@@ -178,7 +178,8 @@ def _oracle_sample(w: wl.Workload, rows: int):
     return np.concatenate(idx_parts).astype(np.int64), off, go
 
 
-def _oracle_rate(w: wl.Workload, budget_s: float, max_rows: int = None):
+def _oracle_rate(w: wl.Workload, budget_s: float, forward_only: bool = False,
+                 max_rows: int = None):
     """Time the CPU oracle (as it stands) on bounded samples of the workload."""
     import oracle
     o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed)
@@ -190,7 +191,8 @@ def _oracle_rate(w: wl.Workload, budget_s: float, max_rows: int = None):
         idx, off, go = _oracle_sample(w, rows)
         t0 = time.perf_counter()
         out, _ = o.forward(wcur, idx, off, rows)
-        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+        if not forward_only:
+            wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
         dt = time.perf_counter() - t0
         if dt > budget_s / 5 or rows >= w.B or (max_rows and rows >= max_rows):
             break
@@ -199,11 +201,27 @@ def _oracle_rate(w: wl.Workload, budget_s: float, max_rows: int = None):
     while tot < budget_s and reps < 20:
         t0 = time.perf_counter()
         out, _ = o.forward(wcur, idx, off, rows)
-        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+        if not forward_only:
+            wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
         tot += time.perf_counter() - t0
         reps += 1
         lookups += idx.shape[0]
     return lookups / tot, rows, reps, idx.shape[0], tot
+
+
+def _shape_overrides(args):
+    """Chunk size Z and offset alignment G given on the command line."""
+    return {k: v for k, v in (("Z", args.Z), ("G", args.G)) if v is not None}
+
+
+def _config_extra(args, w):
+    """Config keys that differ from the named workload's defaults."""
+    extra = {}
+    if args.Z is not None or args.G is not None:
+        extra.update({"Z": w.Z, "G": w.G})
+    if args.forward_only:
+        extra["mode"] = "forward only (inference): hash + gather + sum-pool, no backward"
+    return extra
 
 
 def run_reference(args):
@@ -211,7 +229,7 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    w = wl.make_workload(args.workload, M=args.M, B=args.B)
+    w = wl.make_workload(args.workload, M=args.M, B=args.B, **_shape_overrides(args))
     import oracle
     o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed)
     total_budget = 90.0
@@ -222,28 +240,32 @@ def run_reference(args):
     t0 = time.perf_counter()
     wcur, Gcur = w.w0.copy(), np.zeros(w.M, np.float32)
     o.forward(wcur, idx, off, rows)
-    o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+    if not args.forward_only:
+        o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
     dt = time.perf_counter() - t0
     rows = int(max(1, min(w.B, rows * per_step / max(dt, 1e-6) * 0.8)))
     idx, off, go = _oracle_sample(w, rows)
     for _ in range(args.warmup):
         o.forward(wcur, idx, off, rows)
-        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+        if not args.forward_only:
+            wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
     t0 = time.perf_counter()
     for _ in range(args.steps):
         o.forward(wcur, idx, off, rows)
-        wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
+        if not args.forward_only:
+            wcur, Gcur, _ = o.step(wcur, Gcur, idx, off, rows, go, w.opt, w.lr, w.eps)
     el = time.perf_counter() - t0
     value = idx.shape[0] * args.steps / el
     sample = (f"first {rows} of {w.B} batch rows x {w.T} tables ({idx.shape[0]} lookups) per step; "
-              "forward + gradient + update, single thread")
+              + ("forward only" if args.forward_only else "forward + gradient + update")
+              + ", single thread")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64+f32",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B, "seq_len": 1,
-                   "parallelism": "single host thread"},
+        "config": dict({"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B, "seq_len": 1,
+                        "parallelism": "single host thread"}, **_config_extra(args, w)),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -269,7 +291,7 @@ def run_gpu(args):
         dist.init_process_group("nccl", device_id=dev)
 
     # one replica per rank, each with its own batch (no data-path exchange)
-    w = wl.make_workload(args.workload, seed=0, M=args.M, B=args.B)
+    w = wl.make_workload(args.workload, seed=0, M=args.M, B=args.B, **_shape_overrides(args))
     batches = [(w.indices, w.offsets, w.grad_out)]
     for k in range(1, args.rotate):
         batches.append(wl.make_batch(w.cards, w.B, w.d, wl.CONFIGS[args.workload]["bag"],
@@ -286,8 +308,11 @@ def run_gpu(args):
         h.set_weights(base.repeat(-(-w.M // base.numel()))[: w.M].contiguous())
         del base
     h.set_option(binding.OPT_ACCUM, binding.ACCUM_F32 if args.accum == "f32" else binding.ACCUM_F64)
-    h.set_option(binding.OPT_BACKWARD_PATH, {"auto": binding.PATH_AUTO, "atomic": binding.PATH_ATOMIC,
-                                             "sorted": binding.PATH_SORTED}[args.path])
+    # forward-only: no backward follows, so the forward emits nothing for one
+    h.set_option(binding.OPT_BACKWARD_PATH,
+                 binding.PATH_ATOMIC if args.forward_only else
+                 {"auto": binding.PATH_AUTO, "atomic": binding.PATH_ATOMIC,
+                  "sorted": binding.PATH_SORTED}[args.path])
     out = torch.empty((w.B, w.T, w.d), dtype=torch.float32, device=dev)
     nnz_per_step = [int(b[0].shape[0]) for b in batches]
     stream = torch.cuda.current_stream()
@@ -295,7 +320,8 @@ def run_gpu(args):
     def step(k):
         i, o, g = dbatches[k % len(dbatches)]
         h.forward(i, o, w.B, out=out)
-        h.backward_update(g, w.lr)
+        if not args.forward_only:
+            h.backward_update(g, w.lr)
 
     for k in range(args.warmup):
         step(k)
@@ -360,7 +386,8 @@ def run_gpu(args):
     def step_host(k):
         i, o, g = hb[k % len(hb)]
         h.forward(i, o, w.B, out=hout)
-        h.backward_update(g, w.lr)
+        if not args.forward_only:
+            h.backward_update(g, w.lr)
 
     step_host(0)
     torch.cuda.synchronize()
@@ -380,7 +407,8 @@ def run_gpu(args):
         dist.all_reduce(tmax[:1], op=dist.ReduceOp.MAX)
         dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
         e2e_ms, e2e_lookups = float(tmax[0]), float(t[1])
-    h2d = int(np.mean([i.nbytes + o.nbytes + g.nbytes for i, o, g in batches]))
+    h2d = int(np.mean([i.nbytes + o.nbytes + (0 if args.forward_only else g.nbytes)
+                       for i, o, g in batches]))
     d2h = int(hout.numel() * 4)
 
     if rank == 0:
@@ -396,15 +424,16 @@ def run_gpu(args):
         avg_s = ms_dom / max(1, n_dom) / 1e3
         bytes_dom = ab[dom]
         achieved = bytes_dom / avg_s / 1e9
-        step_bytes = ab["step"]
+        step_bytes = ab["forward"] if args.forward_only else ab["step"]
         step_gbs = step_bytes / (elapsed_ms / args.steps / 1e3) / 1e9 * world
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
-            rate, rows, reps, nnz_s, tot = _oracle_rate(w, args.cpu_budget)
+            rate, rows, reps, nnz_s, tot = _oracle_rate(w, args.cpu_budget, args.forward_only)
             cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                    "sample": (f"first {rows} of {w.B} batch rows x {w.T} tables "
-                              f"({nnz_s} lookups) per step, {reps} steps, {tot:.1f} s: forward + "
-                              "gradient + update, single host thread")}
+                              f"({nnz_s} lookups) per step, {reps} steps, {tot:.1f} s: "
+                              + ("forward only" if args.forward_only else
+                                 "forward + gradient + update") + ", single host thread")}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
@@ -417,7 +446,8 @@ def run_gpu(args):
                        "backward_path": ["auto", "atomic", "sorted"][h.info()["last_path"]],
                        "l2": (f"inputs larger than L2: {args.rotate}-batch rotation, "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB output and "
-                              f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB upstream gradient per step")},
+                              f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB upstream gradient per step"),
+                       **_config_extra(args, w)},
             "step_gbs": step_gbs,
             "bags_per_s": w.B * w.T * args.steps * world / (elapsed_ms / 1e3),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
@@ -462,6 +492,10 @@ def main(argv=None):
     ap.add_argument("--B", type=int, default=None, help="override the batch size (profiling)")
     ap.add_argument("--path", choices=["auto", "atomic", "sorted"], default="auto",
                     help="backward path")
+    ap.add_argument("--Z", type=int, default=None, help="override the chunk size Z")
+    ap.add_argument("--G", type=int, default=None, help="override the offset alignment G")
+    ap.add_argument("--forward-only", action="store_true",
+                    help="time the forward (inference) alone")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")
