@@ -46,7 +46,8 @@ class _Pss(ctypes.Structure):
     _fields_ = [("T", ctypes.c_int64), ("d", ctypes.c_int64), ("M", ctypes.c_int64),
                 ("Z", ctypes.c_int64), ("G", ctypes.c_int64), ("J", ctypes.c_int64),
                 ("L", ctypes.c_int64), ("R", ctypes.c_int64), ("A", ctypes.c_uint64),
-                ("B0", ctypes.c_uint64), ("cards", ctypes.c_void_p)]
+                ("B0", ctypes.c_uint64), ("cards", ctypes.c_void_p), ("sgn", ctypes.c_int64),
+                ("A2", ctypes.c_uint64), ("B2", ctypes.c_uint64)]
 
 
 def _load():
@@ -58,12 +59,16 @@ def _load():
             sig = {
                 "oracle_splitmix64_seq": (None, [u64, i64, vp]),
                 "oracle_hash_params": (None, [u64, vp, vp]),
+                "oracle_sign_params": (None, [u64, vp, vp]),
+                "oracle_set_signed": (None, [vp, i64]),
+                "oracle_sign": (i64, [vp, i64, i64, i64]),
+                "oracle_signs": (ctypes.c_int, [vp, vp, i64, vp, i64, vp]),
                 "oracle_init": (ctypes.c_int, [vp, vp, i64, i64, i64, i64, i64, u64]),
                 "oracle_location": (i64, [vp, i64, i64, i64]),
                 "oracle_locations": (ctypes.c_int, [vp, vp, i64, vp, i64, vp, vp]),
-                "oracle_pool": (ctypes.c_int, [vp, vp, vp, i64, vp, i64, vp]),
+                "oracle_pool": (ctypes.c_int, [vp, vp, vp, i64, vp, i64, vp, vp]),
                 "oracle_forward": (ctypes.c_int, [vp, vp, vp, i64, vp, i64, vp, vp]),
-                "oracle_scatter": (ctypes.c_int, [vp, vp, i64, vp, i64, vp, vp]),
+                "oracle_scatter": (ctypes.c_int, [vp, vp, i64, vp, i64, vp, vp, vp]),
                 "oracle_grad": (ctypes.c_int, [vp, vp, i64, vp, i64, vp, vp, vp]),
                 "oracle_grad_at": (ctypes.c_int, [vp, vp, i64, vp, i64, vp, vp, i64, vp, vp]),
                 "oracle_sgd": (None, [vp, vp, i64, f32]),
@@ -101,11 +106,18 @@ def hash_params(seed: int):
     return int(A.value), int(B0.value)
 
 
+def sign_params(seed: int):
+    A2, B2 = ctypes.c_uint64(), ctypes.c_uint64()
+    _load().oracle_sign_params(ctypes.c_uint64(seed), ctypes.byref(A2), ctypes.byref(B2))
+    return int(A2.value), int(B2.value)
+
+
 class OraclePSS:
     """One PSS instance: T tables, dim d, shared array of M fp32, chunk Z,
     block-start alignment G, hash seed.  All arrays are numpy, host memory."""
 
-    def __init__(self, cards, d: int, M: int, Z: int, G: int = 4, seed: int = 0):
+    def __init__(self, cards, d: int, M: int, Z: int, G: int = 4, seed: int = 0,
+                 signed: bool = False):
         self._lib = _load()
         self.cards = _c(cards, np.int64)
         self.T = int(self.cards.shape[0])
@@ -117,6 +129,9 @@ class OraclePSS:
             raise OracleError(f"oracle_init failed ({rc})")
         self.J, self.L, self.R = int(self._p.J), int(self._p.L), int(self._p.R)
         self.A, self.B0 = int(self._p.A), int(self._p.B0)
+        self.A2, self.B2 = int(self._p.A2), int(self._p.B2)
+        self.signed = bool(signed)
+        self._lib.oracle_set_signed(ctypes.byref(self._p), 1 if signed else 0)
 
     def _pp(self):
         return ctypes.byref(self._p)
@@ -134,10 +149,25 @@ class OraclePSS:
             raise OracleError(f"oracle_locations failed ({rc})")
         return locs[: idx.shape[0] * self.J], int(bad.value)
 
-    def pool(self, w, locs, offsets, B: int, nnz: int):
+    def sign(self, i: int, t: int, j: int) -> int:
+        """+1, or -1 for a key with an odd sign hash when signed hashing is on."""
+        return int(self._lib.oracle_sign(self._pp(), i, t, j))
+
+    def signs(self, indices, offsets, B: int):
+        """Sign of every (id, chunk), laid out like locations (0 for a bad id)."""
+        idx, off = _c(indices, np.int64), _c(offsets, np.int64)
+        sg = np.zeros(max(1, idx.shape[0] * self.J), dtype=np.int8)
+        rc = self._lib.oracle_signs(self._pp(), _ptr(idx), idx.shape[0], _ptr(off), B, _ptr(sg))
+        if rc:
+            raise OracleError(f"oracle_signs failed ({rc})")
+        return sg[: idx.shape[0] * self.J]
+
+    def pool(self, w, locs, offsets, B: int, nnz: int, signs=None):
         w, locs, off = _c(w, np.float32), _c(locs, np.int64), _c(offsets, np.int64)
         out = np.zeros(B * self.T * self.d, dtype=np.float32)
-        rc = self._lib.oracle_pool(self._pp(), _ptr(w), _ptr(locs), nnz, _ptr(off), B, _ptr(out))
+        sg = None if signs is None else _c(signs, np.int8)
+        rc = self._lib.oracle_pool(self._pp(), _ptr(w), _ptr(locs), nnz, _ptr(off), B, _ptr(out),
+                                   None if sg is None else _ptr(sg))
         if rc:
             raise OracleError(f"oracle_pool failed ({rc})")
         return out
@@ -152,10 +182,12 @@ class OraclePSS:
             raise OracleError(f"oracle_forward failed ({rc})")
         return out, int(bad.value)
 
-    def scatter(self, locs, offsets, B: int, nnz: int, grad_out):
+    def scatter(self, locs, offsets, B: int, nnz: int, grad_out, signs=None):
         locs, off, go = _c(locs, np.int64), _c(offsets, np.int64), _c(grad_out, np.float32)
         g = np.zeros(self.M, dtype=np.float64)
-        rc = self._lib.oracle_scatter(self._pp(), _ptr(locs), nnz, _ptr(off), B, _ptr(go), _ptr(g))
+        sg = None if signs is None else _c(signs, np.int8)
+        rc = self._lib.oracle_scatter(self._pp(), _ptr(locs), nnz, _ptr(off), B, _ptr(go), _ptr(g),
+                                      None if sg is None else _ptr(sg))
         if rc:
             raise OracleError(f"oracle_scatter failed ({rc})")
         return g

@@ -34,7 +34,13 @@
  *     B0 = s2 mod P;
  *   - sums are taken in fp64 and rounded to fp32 once; the optimizer update is
  *     done in fp32, one IEEE operation at a time in a fixed order (compile
- *     with -ffp-contract=off so no multiply-add is fused).
+ *     with -ffp-contract=off so no multiply-add is fused);
+ *   - signed hashing (optional; Sec. 2.5 derives the sketch from Achlioptas'
+ *     +-1 random projections, ROBE-Z itself has no sign): every (id, chunk)
+ *     also gets a sign s = +-1 from a second hash of the same family with its
+ *     own parameters A2 = 1 + (s3 mod (P-1)), B2 = s4 mod P (the third and
+ *     fourth splitmix64 outputs): s = -1 when (A2*key + B2) mod P is odd.  The
+ *     forward adds s * block, the backward adds s * upstream gradient.
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -48,6 +54,8 @@ typedef struct {
     int64_t J, L, R;              /* chunks per embedding, block length read, #starts */
     uint64_t A, B0;               /* hash parameters */
     const int64_t* cards;         /* host, T cardinalities (not owned) */
+    int64_t sgn;                  /* 1: signed hashing */
+    uint64_t A2, B2;              /* sign-hash parameters */
 } oracle_pss;
 
 /* splitmix64 (Steele, Lea & Flood, "Fast splittable pseudorandom number
@@ -81,6 +89,18 @@ void oracle_hash_params(uint64_t seed, uint64_t* A, uint64_t* B0)
     *B0 = s2 % ORACLE_P;
 }
 
+/* Sign-hash parameters: the third and fourth splitmix64 outputs of the seed. */
+void oracle_sign_params(uint64_t seed, uint64_t* A2, uint64_t* B2)
+{
+    uint64_t s = seed, s3, s4;
+    oracle_splitmix64(&s);
+    oracle_splitmix64(&s);
+    s3 = oracle_splitmix64(&s);
+    s4 = oracle_splitmix64(&s);
+    *A2 = 1 + (s3 % (ORACLE_P - 1));
+    *B2 = s4 % ORACLE_P;
+}
+
 /* Set up one PSS instance.  Returns 0 on success, a negative code when the
  * sizes are invalid (no block fits, or keys would exceed the hash's field). */
 int oracle_init(oracle_pss* p, const int64_t* cards, int64_t T, int64_t d, int64_t M,
@@ -102,7 +122,15 @@ int oracle_init(oracle_pss* p, const int64_t* cards, int64_t T, int64_t d, int64
         > (unsigned __int128)ORACLE_P) return -4;
     p->cards = cards;
     oracle_hash_params(seed, &p->A, &p->B0);
+    oracle_sign_params(seed, &p->A2, &p->B2);
+    p->sgn = 0;
     return 0;
+}
+
+/* Turn signed hashing on (1) or off (0). */
+void oracle_set_signed(oracle_pss* p, int64_t on)
+{
+    p->sgn = on ? 1 : 0;
 }
 
 /* h(t, i, j): start of the block that holds chunk j of id i of table t
@@ -113,6 +141,18 @@ int64_t oracle_location(const oracle_pss* p, int64_t id, int64_t t, int64_t j)
     unsigned __int128 v = (unsigned __int128)p->A * key + p->B0;
     uint64_t x = (uint64_t)(v % ORACLE_P);
     return p->G * (int64_t)(x % (uint64_t)p->R);
+}
+
+/* s(t, i, j): +1, or -1 when signed hashing is on and the sign hash of the
+ * key is odd. */
+int64_t oracle_sign(const oracle_pss* p, int64_t id, int64_t t, int64_t j)
+{
+    uint64_t key;
+    unsigned __int128 v;
+    if (!p->sgn) return 1;
+    key = ((uint64_t)id * (uint64_t)p->T + (uint64_t)t) * (uint64_t)p->J + (uint64_t)j;
+    v = (unsigned __int128)p->A2 * key + p->B2;
+    return ((uint64_t)(v % ORACLE_P) & 1u) ? -1 : 1;
 }
 
 /* Check the CSR bag layout: offsets non-decreasing, inside [0, nnz]. */
@@ -153,11 +193,33 @@ int oracle_locations(const oracle_pss* p, const int64_t* indices, int64_t nnz,
     return 0;
 }
 
+/* Signs of every (id, chunk), laid out like the locations: signs[q*J + j] =
+ * s(t, indices[q], j), 0 for an id outside its table. */
+int oracle_signs(const oracle_pss* p, const int64_t* indices, int64_t nnz,
+                 const int64_t* offsets, int64_t B, int8_t* signs)
+{
+    int rc = check_offsets(offsets, p->T * B, nnz);
+    if (rc) return rc;
+    for (int64_t q = 0; q < nnz * p->J; ++q) signs[q] = 0;
+    for (int64_t t = 0; t < p->T; ++t)
+        for (int64_t b = 0; b < B; ++b) {
+            int64_t s = t * B + b;
+            for (int64_t q = offsets[s]; q < offsets[s + 1]; ++q) {
+                int64_t id = indices[q];
+                if (id < 0 || id >= p->cards[t]) continue;
+                for (int64_t j = 0; j < p->J; ++j)
+                    signs[q * p->J + j] = (int8_t)oracle_sign(p, id, t, j);
+            }
+        }
+    return 0;
+}
+
 /* Sum-pooled forward from given locations (Sec. 2.4 forward, summed over the
- * ids of a bag): out[b][t][jZ+z] = sum_q M[locs[q*J+j] + z], z < min(Z, d-jZ).
+ * ids of a bag): out[b][t][jZ+z] = sum_q s_qj * M[locs[q*J+j] + z],
+ * z < min(Z, d-jZ), with s_qj = signs[q*J+j] (+1 when signs is NULL).
  * An empty bag gives zeros; an entry with loc < 0 contributes nothing. */
 int oracle_pool(const oracle_pss* p, const float* w, const int64_t* locs, int64_t nnz,
-                const int64_t* offsets, int64_t B, float* out)
+                const int64_t* offsets, int64_t B, float* out, const int8_t* signs)
 {
     int64_t d = p->d, T = p->T;
     double* acc;
@@ -173,8 +235,9 @@ int oracle_pool(const oracle_pss* p, const float* w, const int64_t* locs, int64_
                 for (int64_t j = 0; j < p->J; ++j) {
                     int64_t loc = locs[q * p->J + j];
                     int64_t Lj = d - j * p->Z < p->Z ? d - j * p->Z : p->Z;
+                    double sg = signs ? (double)signs[q * p->J + j] : 1.0;
                     if (loc < 0) continue;
-                    for (int64_t z = 0; z < Lj; ++z) acc[j * p->Z + z] += (double)w[loc + z];
+                    for (int64_t z = 0; z < Lj; ++z) acc[j * p->Z + z] += sg * (double)w[loc + z];
                 }
             for (int64_t k = 0; k < d; ++k) out[(b * T + t) * d + k] = (float)acc[k];
         }
@@ -182,25 +245,34 @@ int oracle_pool(const oracle_pss* p, const float* w, const int64_t* locs, int64_
     return 0;
 }
 
-/* Forward pass: hash every (id, chunk), then gather and sum-pool. */
+/* Forward pass: hash every (id, chunk) (and sign it, when signed hashing is
+ * on), then gather and sum-pool. */
 int oracle_forward(const oracle_pss* p, const float* w, const int64_t* indices, int64_t nnz,
                    const int64_t* offsets, int64_t B, float* out, int64_t* first_bad)
 {
     int64_t* locs = (int64_t*)malloc(sizeof(int64_t) * (size_t)(nnz * p->J + 1));
+    int8_t* signs = p->sgn ? (int8_t*)malloc((size_t)(nnz * p->J + 1)) : NULL;
     int rc;
-    if (!locs) return -20;
+    if (!locs || (p->sgn && !signs)) {
+        free(locs);
+        free(signs);
+        return -20;
+    }
     rc = oracle_locations(p, indices, nnz, offsets, B, locs, first_bad);
-    if (!rc) rc = oracle_pool(p, w, locs, nnz, offsets, B, out);
+    if (!rc && signs) rc = oracle_signs(p, indices, nnz, offsets, B, signs);
+    if (!rc) rc = oracle_pool(p, w, locs, nnz, offsets, B, out, signs);
     free(locs);
+    free(signs);
     return rc;
 }
 
 /* Dense branch of Algorithm 1 from given locations: g (length M, fp64,
  * zeroed here) receives, for every bag, id and chunk, the upstream gradient of
- * that bag's output chunk added element by element at the block's location
+ * that bag's output chunk, times the chunk's sign (signs[q*J+j], +1 when
+ * signs is NULL), added element by element at the block's location
  * (Sec. 2.4 backward(i, D) = (S e_i) D, summed over the ids of each bag). */
 int oracle_scatter(const oracle_pss* p, const int64_t* locs, int64_t nnz, const int64_t* offsets,
-                   int64_t B, const float* grad_out, double* g)
+                   int64_t B, const float* grad_out, double* g, const int8_t* signs)
 {
     int64_t d = p->d, T = p->T;
     int rc = check_offsets(offsets, T * B, nnz);
@@ -214,8 +286,9 @@ int oracle_scatter(const oracle_pss* p, const int64_t* locs, int64_t nnz, const 
                 for (int64_t j = 0; j < p->J; ++j) {
                     int64_t loc = locs[q * p->J + j];
                     int64_t Lj = d - j * p->Z < p->Z ? d - j * p->Z : p->Z;
+                    double sg = signs ? (double)signs[q * p->J + j] : 1.0;
                     if (loc < 0) continue;
-                    for (int64_t z = 0; z < Lj; ++z) g[loc + z] += (double)go[j * p->Z + z];
+                    for (int64_t z = 0; z < Lj; ++z) g[loc + z] += sg * (double)go[j * p->Z + z];
                 }
         }
     return 0;
@@ -226,11 +299,18 @@ int oracle_grad(const oracle_pss* p, const int64_t* indices, int64_t nnz, const 
                 int64_t B, const float* grad_out, double* g, int64_t* first_bad)
 {
     int64_t* locs = (int64_t*)malloc(sizeof(int64_t) * (size_t)(nnz * p->J + 1));
+    int8_t* signs = p->sgn ? (int8_t*)malloc((size_t)(nnz * p->J + 1)) : NULL;
     int rc;
-    if (!locs) return -20;
+    if (!locs || (p->sgn && !signs)) {
+        free(locs);
+        free(signs);
+        return -20;
+    }
     rc = oracle_locations(p, indices, nnz, offsets, B, locs, first_bad);
-    if (!rc) rc = oracle_scatter(p, locs, nnz, offsets, B, grad_out, g);
+    if (!rc && signs) rc = oracle_signs(p, indices, nnz, offsets, B, signs);
+    if (!rc) rc = oracle_scatter(p, locs, nnz, offsets, B, grad_out, g, signs);
     free(locs);
+    free(signs);
     return rc;
 }
 
@@ -267,9 +347,10 @@ int oracle_grad_at(const oracle_pss* p, const int64_t* indices, int64_t nnz, con
                 for (int64_t j = 0; j < p->J; ++j) {
                     int64_t loc = oracle_location(p, id, t, j);
                     int64_t Lj = d - j * p->Z < p->Z ? d - j * p->Z : p->Z;
+                    double sg = (double)oracle_sign(p, id, t, j);
                     for (int64_t k = lower_bound_i64(elems, n_elems, loc);
                          k < n_elems && elems[k] < loc + Lj; ++k)
-                        g_at[k] += (double)go[j * p->Z + (elems[k] - loc)];
+                        g_at[k] += sg * (double)go[j * p->Z + (elems[k] - loc)];
                 }
             }
         }

@@ -155,6 +155,86 @@ def test_forward_and_grad_equal_bruteforce_matrix(Z, G, d):
         np.testing.assert_array_equal(g, P.T @ go.astype(np.float64))
 
 
+# --------------------------------------------------------------------------
+# signed hashing: every (id, chunk) also carries a sign s = +-1 from a second
+# hash of the same family (Sec. 2.5: the sketch comes from +-1 projections)
+@pytest.mark.parametrize("seed", [0, 7, 2**63 + 7])
+def test_sign_hash_matches_bigint(seed):
+    cards = [1000, 37, 40_000_000]
+    o = OraclePSS(cards, d=128, M=2_500_000, Z=32, G=4, seed=seed, signed=True)
+    A2, B2 = bh.sign_params(seed)
+    assert (o.A2, o.B2) == (A2, B2)
+    assert (o.A, o.B0) != (o.A2, o.B2)
+    rng = np.random.default_rng(seed % 1000)
+    for _ in range(300):
+        t = int(rng.integers(0, 3))
+        i = int(rng.integers(0, cards[t]))
+        j = int(rng.integers(0, o.J))
+        assert o.sign(i, t, j) == bh.sign(A2, B2, 3, o.J, i, t, j)
+    # unsigned instance: every sign is +1
+    u = OraclePSS(cards, d=128, M=2_500_000, Z=32, G=4, seed=seed)
+    assert all(u.sign(i, 0, 0) == 1 for i in range(50))
+
+
+def test_signs_are_balanced():
+    o = OraclePSS([10_000_000] * 4, d=128, M=2_500_000, Z=32, G=4, seed=3, signed=True)
+    s = np.array([o.sign(i, t, j) for i in range(0, 4000, 3) for t in range(4) for j in range(4)])
+    n = s.shape[0]
+    # a fair coin: the count of -1 within 5 standard deviations of n/2
+    assert abs((s == -1).sum() - n / 2) < 5 * np.sqrt(n / 4)
+
+
+@pytest.mark.parametrize("Z,G,d", [(1, 1, 16), (4, 4, 16), (32, 4, 16), (3, 2, 10)])
+def test_signed_forward_and_grad_equal_signed_bruteforce_matrix(Z, G, d):
+    # the explicit +-1 mapping matrix from big integers: forward = P w and
+    # gradient = P^T g, bit for bit on dyadic inputs
+    T, B, M = 2, 4, 256
+    for seed in range(3):
+        cards, idx, off, w, go = _tiny_case(seed, T=T, B=B, d=d, M=M, Z=Z, G=G)
+        o = OraclePSS(cards, d=d, M=M, Z=Z, G=G, seed=seed, signed=True)
+        A, B0 = bh.params(seed)
+        A2, B2 = bh.sign_params(seed)
+        L, J = min(Z, d), -(-d // Z)
+        R = (M - L) // G + 1
+        rows, cols, vals = [], [], []
+        for t in range(T):
+            for b in range(B):
+                s = t * B + b
+                for q in range(off[s], off[s + 1]):
+                    i = int(idx[q])
+                    for k in range(d):
+                        j, z = divmod(k, Z)
+                        rows.append((b * T + t) * d + k)
+                        cols.append(bh.location(A, B0, R, G, T, J, i, t, j) + z)
+                        vals.append(bh.sign(A2, B2, T, J, i, t, j))
+        P = sp.coo_matrix((vals, (rows, cols)), shape=(B * T * d, M)).tocsr()
+        out, bad = o.forward(w, idx, off, B)
+        assert bad == -1
+        np.testing.assert_array_equal(out, (P @ w.astype(np.float64)).astype(np.float32))
+        np.testing.assert_array_equal(o.grad(idx, off, B, go), P.T @ go.astype(np.float64))
+
+
+@pytest.mark.parametrize("signed", [False, True])
+def test_backward_is_the_adjoint_of_the_forward(signed):
+    # <forward(w), g> == <w, grad(g)> for any w, g: the backward of Sec. 2.4 is
+    # the transpose of the forward, with or without signs (dyadic: exact)
+    cards, idx, off, w, go = _tiny_case(11, T=3, B=8, d=16, M=300, Z=4, G=1, max_bag=5)
+    o = OraclePSS(cards, d=16, M=300, Z=4, G=1, seed=5, signed=signed)
+    out, _ = o.forward(w, idx, off, 8)
+    g = o.grad(idx, off, 8, go)
+    lhs = float(np.dot(out.astype(np.float64), go.astype(np.float64)))
+    rhs = float(np.dot(w.astype(np.float64), g))
+    assert lhs == rhs
+
+
+def test_signed_grad_at_matches_signed_dense_grad():
+    cards, idx, off, w, go = _tiny_case(4, T=2, B=6, d=16, M=512, Z=4, G=2, max_bag=4, dy=False)
+    o = OraclePSS(cards, d=16, M=512, Z=4, G=2, seed=8, signed=True)
+    g = o.grad(idx, off, 6, go)
+    elems = np.flatnonzero(g)
+    np.testing.assert_array_equal(o.grad_at(idx, off, 6, go, elems), g[elems])
+
+
 def test_forward_bruteforce_non_dyadic():
     cards, idx, off, w, go = _tiny_case(5, T=3, B=8, d=16, M=300, Z=4, G=1, max_bag=6, dy=False)
     o = OraclePSS(cards, d=16, M=300, Z=4, G=1, seed=9)
