@@ -221,6 +221,8 @@ def _config_extra(args, w):
         extra.update({"Z": w.Z, "G": w.G})
     if args.forward_only:
         extra["mode"] = "forward only (inference): hash + gather + sum-pool, no backward"
+    if args.signed:
+        extra["signed_hash"] = True
     return extra
 
 
@@ -231,7 +233,7 @@ def run_reference(args):
         return 0
     w = wl.make_workload(args.workload, M=args.M, B=args.B, **_shape_overrides(args))
     import oracle
-    o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed)
+    o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, signed=args.signed)
     total_budget = 90.0
     per_step = total_budget / max(1, args.steps + args.warmup)
     # size the per-step sample so K+W steps fit the budget
@@ -308,6 +310,8 @@ def run_gpu(args):
         h.set_weights(base.repeat(-(-w.M // base.numel()))[: w.M].contiguous())
         del base
     h.set_option(binding.OPT_ACCUM, binding.ACCUM_F32 if args.accum == "f32" else binding.ACCUM_F64)
+    if args.signed:
+        h.set_option(binding.OPT_SIGNED, 1)
     # forward-only: no backward follows, so the forward emits nothing for one
     h.set_option(binding.OPT_BACKWARD_PATH,
                  binding.PATH_ATOMIC if args.forward_only else
@@ -496,6 +500,7 @@ def main(argv=None):
     ap.add_argument("--G", type=int, default=None, help="override the offset alignment G")
     ap.add_argument("--forward-only", action="store_true",
                     help="time the forward (inference) alone")
+    ap.add_argument("--signed", action="store_true", help="signed hashing (PSS_OPT_SIGNED)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")

@@ -103,7 +103,19 @@ typedef enum {
      * PSS_ACCUM_F32: 16-byte fp32 vector reductions (4 bytes per element, and
      * SGD is scattered straight into M); the error of a recursive fp32 sum,
      * up to (n-1) * 2^-24 * sum|contributions| for an element with n of them. */
-    PSS_OPT_ACCUM = 5
+    PSS_OPT_ACCUM = 5,
+    /* 1: signed hashing.  Every (table t, id i, chunk j) also gets a sign
+     * s = +-1 from a second hash of the same family (Sec. 2.5 builds the sketch
+     * from +-1 random projections; ROBE-Z itself has none):
+     *   s = -1 when ((A2*key + B2) mod (2^61-1)) is odd, else +1,
+     * key as for the location, A2 = 1 + (s3 mod (2^61-2)) and B2 = s4 mod
+     * (2^61-1) from the third and fourth splitmix64 outputs of the seed.  The
+     * forward adds s * block and the backward s * upstream gradient.
+     * Needs R < 2^31 (PSS_ERR_UNSUPPORTED otherwise).  Changing it forgets the
+     * last forward's batch (the next backward needs a new forward).
+     * pss_compute_locations returns locations only; pss_grad_noalloc is
+     * unsigned. */
+    PSS_OPT_SIGNED = 6
 } pss_option;
 
 
@@ -119,8 +131,8 @@ typedef enum {
     PSS_K_FORWARD = 1,     /* fused hash + gather + sum-pool */
     PSS_K_SCATTER = 2,     /* backward: hash + vector-atomic scatter (+ fused SGD) */
     PSS_K_UPDATE = 3,      /* optimizer pass over M (dense or touched blocks) */
-    PSS_K_SORT = 4,        /* sorted path: key build + radix sort passes */
-    PSS_K_REDUCE = 5,      /* sorted path: segmented reduce + fused update */
+    PSS_K_SORT = 4,        /* sorted path: bucket count, scan and slot scatter */
+    PSS_K_REDUCE = 5,      /* sorted path: run sums into the fp64 accumulator */
     PSS_K_MISC = 6,        /* memsets and small helper kernels */
     PSS_K_COUNT = 7
 } pss_kernel_id;
@@ -133,6 +145,8 @@ typedef struct {
     int64_t kernel_launches;   /* kernels this handle has launched so far */
     int64_t last_path;         /* PSS_PATH_ATOMIC / PSS_PATH_SORTED of the last backward */
     double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass, or -1 */
+    uint64_t A2, B2;           /* sign-hash parameters derived from the seed */
+    int64_t signed_hash;       /* PSS_OPT_SIGNED */
 } pss_info;
 
 /*

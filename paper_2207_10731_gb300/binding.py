@@ -23,6 +23,7 @@ PSS_OK, PSS_ERR_INVALID_ARG, PSS_ERR_OOM, PSS_ERR_CUDA, PSS_ERR_STATE, PSS_ERR_I
     PSS_ERR_TIMEOUT, PSS_ERR_UNSUPPORTED, PSS_ERR_CAPACITY = range(9)
 PSS_SGD, PSS_ADAGRAD = 0, 1
 OPT_BACKWARD_PATH, OPT_UPDATE_MODE, OPT_PROFILE, OPT_SYNC_CHECK, OPT_ACCUM = 1, 2, 3, 4, 5
+OPT_SIGNED = 6
 ACCUM_F64, ACCUM_F32 = 0, 1
 PATH_AUTO, PATH_ATOMIC, PATH_SORTED = 0, 1, 2
 UPDATE_AUTO, UPDATE_DENSE, UPDATE_TOUCHED = 0, 1, 2
@@ -45,7 +46,8 @@ class PSSInfo(ctypes.Structure):
                 ("L", ctypes.c_int64), ("R", ctypes.c_int64), ("A", ctypes.c_uint64),
                 ("B0", ctypes.c_uint64), ("optimizer", ctypes.c_int64),
                 ("kernel_launches", ctypes.c_int64), ("last_path", ctypes.c_int64),
-                ("last_collision_rate", ctypes.c_double)]
+                ("last_collision_rate", ctypes.c_double), ("A2", ctypes.c_uint64),
+                ("B2", ctypes.c_uint64), ("signed_hash", ctypes.c_int64)]
 
 
 class PSSError(RuntimeError):

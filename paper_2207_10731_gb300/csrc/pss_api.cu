@@ -298,8 +298,11 @@ constexpr int64_t kAutoSortedMaxR = int64_t(1) << 26;
 
 bool sorted_supported(const pss_handle* h, int64_t nnz, int64_t B) {
     const int64_t J = h->dp.J;
+    // entries hold row*J + j in 32 bits (31 with signed hashing: the sign
+    // travels in bit 31)
+    const int64_t lim = h->dp.smask ? (int64_t)0x7fffffffLL : (int64_t)0xffffffffLL;
     return (int64_t)h->dp.R <= kSortedMaxR && nnz * J < (int64_t)0xffffffffLL &&
-           (int64_t)h->dp.T * B * J < (int64_t)0xffffffffLL;
+           (int64_t)h->dp.T * B * J < lim;
 }
 
 bool want_sorted(const pss_handle* h) {
@@ -442,10 +445,13 @@ pss_status pss_create(const int64_t* cards, int32_t T, int32_t dim, int64_t M, i
         return z ^ (z >> 31);
     };
     const uint64_t p61 = (uint64_t(1) << 61) - 1;
-    const uint64_t s1 = next(), s2 = next();
+    const uint64_t s1 = next(), s2 = next(), s3 = next(), s4 = next();
     DevParams& dp = h->dp;
     dp.A = 1 + s1 % (p61 - 1);
     dp.B0 = s2 % p61;
+    dp.A2 = 1 + s3 % (p61 - 1);
+    dp.B2 = s4 % p61;
+    dp.smask = 0u;
     dp.G = G;
     dp.M = M;
     dp.T = T;
@@ -662,9 +668,9 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, 
     // scatter counts each bucket back down by exactly what its count added
     {
         LaunchScope ls(h, PSS_K_SORT, st, 5);
-        PSS_TRY(launch_sorted_count(h->sb, npairs, h->sm_count, st));
+        PSS_TRY(launch_sorted_count(h->sb, npairs, h->dp.smask, h->sm_count, st));
         PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, touch ? &h->touched : nullptr, st));
-        PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->sm_count, st));
+        PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->dp.smask, h->sm_count, st));
     }
     if (!h->stats_pending) {
         PSS_TRY(cudaMemcpyAsync(h->stats_host, h->sb.stats, 2 * sizeof(unsigned long long),
@@ -826,6 +832,15 @@ pss_status pss_set_option(pss_handle* h, int32_t key, int64_t value) {
             if (value != PSS_ACCUM_F64 && value != PSS_ACCUM_F32) return PSS_ERR_INVALID_ARG;
             h->accum = value;
             return PSS_OK;
+        case PSS_OPT_SIGNED: {
+            if (value != 0 && value != 1) return PSS_ERR_INVALID_ARG;
+            // the sign travels in bit 31 of a 32-bit bucket index
+            if (value && h->dp.R >= (uint64_t(1) << 31)) return PSS_ERR_UNSUPPORTED;
+            const uint32_t m = value ? 0x80000000u : 0u;
+            if (m != h->dp.smask) h->have_batch = false;
+            h->dp.smask = m;
+            return PSS_OK;
+        }
     }
     return PSS_ERR_INVALID_ARG;
 }
@@ -838,6 +853,7 @@ pss_status pss_get_option(pss_handle* h, int32_t key, int64_t* value) {
         case PSS_OPT_PROFILE: *value = h->profile; return PSS_OK;
         case PSS_OPT_SYNC_CHECK: *value = h->sync_check; return PSS_OK;
         case PSS_OPT_ACCUM: *value = h->accum; return PSS_OK;
+        case PSS_OPT_SIGNED: *value = h->dp.smask ? 1 : 0; return PSS_OK;
     }
     return PSS_ERR_INVALID_ARG;
 }
@@ -861,6 +877,9 @@ pss_status pss_get_info(pss_handle* h, pss_info* info) {
     info->R = (int64_t)h->dp.R;
     info->A = h->dp.A;
     info->B0 = h->dp.B0;
+    info->A2 = h->dp.A2;
+    info->B2 = h->dp.B2;
+    info->signed_hash = h->dp.smask ? 1 : 0;
     info->optimizer = h->opt;
     info->kernel_launches = h->launches;
     info->last_path = h->last_path;

@@ -15,13 +15,17 @@ constexpr uint64_t kP61 = (uint64_t(1) << 61) - 1;
 // A*key < 2^122 is folded with 2^61 == 1 (mod P); "mod R" uses the
 // precomputed Rinv = floor((2^64-1)/R): q' = umulhi(s, Rinv) is q or q-1 for
 // s < 2^64 (Barrett, CRYPTO '86), so one conditional subtraction is exact.
-__device__ __forceinline__ uint64_t hash_bucket(const DevParams& p, uint64_t key) {
-    const uint64_t lo = p.A * key;
-    const uint64_t hi = __umul64hi(p.A, key);            // < 2^58
+__device__ __forceinline__ uint64_t affine_mod_p61(uint64_t a, uint64_t key, uint64_t b) {
+    const uint64_t lo = a * key;
+    const uint64_t hi = __umul64hi(a, key);               // < 2^58
     uint64_t s = (lo & kP61) + ((lo >> 61) | (hi << 3));  // < 2^62
-    s += p.B0;                                            // < 2^62 + 2^61
+    s += b;                                               // < 2^62 + 2^61
     s = (s & kP61) + (s >> 61);                           // < 2^61 + 3
-    s = (s >= kP61) ? s - kP61 : s;
+    return (s >= kP61) ? s - kP61 : s;
+}
+
+__device__ __forceinline__ uint64_t hash_bucket(const DevParams& p, uint64_t key) {
+    const uint64_t s = affine_mod_p61(p.A, key, p.B0);
     const uint64_t q = __umul64hi(s, p.Rinv);
     uint64_t r = s - q * p.R;
     return (r >= p.R) ? r - p.R : r;
@@ -29,6 +33,24 @@ __device__ __forceinline__ uint64_t hash_bucket(const DevParams& p, uint64_t key
 
 __device__ __forceinline__ uint64_t hash_key(const DevParams& p, uint64_t id, int t, int j) {
     return (id * (uint64_t)p.T + (uint64_t)t) * (uint64_t)p.J + (uint64_t)j;
+}
+
+// Signed hashing: the sign s = -1 of a key whose sign hash (A2*key + B2) mod
+// (2^61-1) is odd, as the fp32 sign bit (0x80000000); 0 for s = +1 and
+// whenever signed hashing is off (smask == 0).  Bucket indices carry it in
+// their bit 31 (R < 2^31 with signed hashing), which is where fp32 keeps its
+// sign, so a value is signed by an XOR with the index's masked bit.
+__device__ __forceinline__ uint32_t hash_sign_bit(const DevParams& p, uint64_t key) {
+    if (!p.smask) return 0u;
+    return (uint32_t)(affine_mod_p61(p.A2, key, p.B2) & 1u) << 31;
+}
+
+__device__ __forceinline__ float sign_by(float v, uint32_t sbit) {
+    return __uint_as_float(__float_as_uint(v) ^ sbit);
+}
+__device__ __forceinline__ float4 sign_by(float4 v, uint32_t sbit) {
+    return make_float4(sign_by(v.x, sbit), sign_by(v.y, sbit), sign_by(v.z, sbit),
+                       sign_by(v.w, sbit));
 }
 
 __device__ __forceinline__ void record_bad_id(DevError* err, int64_t q) {

@@ -15,6 +15,8 @@ struct DevParams {
     int64_t G, M;
     int32_t T, d, Z, J, L;
     const int64_t* cards;   // device, T entries
+    uint64_t A2, B2;        // sign hash
+    uint32_t smask;         // 0x80000000 with signed hashing, else 0 (see pss_device.cuh)
 };
 
 // Device error word: smallest id position seen out of range, and flag bits.
@@ -54,13 +56,13 @@ struct SortedBuffers {
 };
 int64_t sorted_scan_blocks(int64_t R);
 // Per-bucket counts of the valid pairs (cnt must be zero on entry).
-cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, int sm_count,
-                                cudaStream_t st);
+cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
+                                int sm_count, cudaStream_t st);
 // Bucket starts; with `touched`, also the list / bitmap of non-empty buckets.
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
                                cudaStream_t st);
-cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
-                                  cudaStream_t st);
+cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
+                                  int sm_count, cudaStream_t st);
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
                                  const DevParams& p, double* g, int sm_count, cudaStream_t st);
 

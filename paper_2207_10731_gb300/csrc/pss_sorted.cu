@@ -12,7 +12,8 @@
 //               statistics: valid pairs and distinct buckets;
 //   2. scatter  each pair takes a slot in [start[x], start[x+1]) of sorted_e,
 //               which holds (x, r = row*J + j): the bucket and the
-//               upstream-gradient chunk to add;
+//               upstream-gradient chunk to add (with signed hashing, bit 31 of
+//               pair_x and of r carries the pair's sign, see pss_device.cuh);
 //   3. reduce   the sorted entries are cut into tasks of kPiece consecutive
 //               entries; one group of lanes per task owns 16-byte columns of
 //               the block, adds the chunks of each run of equal x with
@@ -203,7 +204,8 @@ __device__ __forceinline__ void seg_table_init(uint32_t* s_key, uint32_t* s_val)
 
 // cnt[x] += number of valid pairs with bucket x.
 __global__ void __launch_bounds__(kSegThreads)
-k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t* __restrict__ cnt) {
+k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask,
+             uint32_t* __restrict__ cnt) {
     pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
     __shared__ uint32_t s_val[kSegSlots];
@@ -220,7 +222,7 @@ k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t* __re
         __syncthreads();   // the previous segment's table is clear
 #pragma unroll
         for (int i = 0; i < kSegPer; ++i)
-            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i]) : 0u;
+            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i] & ~smask) : 0u;
         __syncthreads();
 #pragma unroll
         for (int k = 0; k < kSegSlots / kSegThreads; ++k) {
@@ -243,10 +245,11 @@ k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t* __re
 // one contiguous range of every bucket it holds (one atomic per distinct
 // bucket); within the range a pair's place is its rank in the segment table.
 // sorted_e[slot] = x << 32 | row*J + j.
+template <bool SG>
 __global__ void __launch_bounds__(kSegThreads)
 k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
-               int J, int log2J, const uint32_t* __restrict__ start, uint32_t* __restrict__ cnt,
-               unsigned long long* __restrict__ sorted_e) {
+               int J, int log2J, const uint32_t* __restrict__ start,
+               uint32_t* __restrict__ cnt, unsigned long long* __restrict__ sorted_e) {
     pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
     __shared__ uint32_t s_val[kSegSlots];
@@ -269,6 +272,11 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
             st0[i] = 0u;
             if (x[i] != kBad) {
                 e[i] += __ldg(q_row + q) * (uint32_t)J;
+                if (SG) {
+                    // signed hashing: the sign moves to bit 31 of the entry's low word
+                    e[i] |= x[i] & 0x80000000u;
+                    x[i] &= 0x7fffffffu;
+                }
                 st0[i] = __ldg(start + x[i]);
             }
         }
@@ -324,7 +332,7 @@ __global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
 k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                const unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
-               double* __restrict__ g, int log2gs) {
+               uint32_t smask, double* __restrict__ g, int log2gs) {
     pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
@@ -389,14 +397,15 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
             for (int u = 0; u < kRU; ++u) {
                 xs[u] = (uint32_t)(ent[u] >> 32);
-                const uint32_t r = (uint32_t)ent[u];
+                const uint32_t r = (uint32_t)ent[u] & ~smask;
+                const uint32_t sb = (uint32_t)ent[u] & smask;
                 if (xs[u] != kBad) {
                     if (ZDIV) {
                         // Z divides d: chunk r starts at r*Z and is Z long
                         const float* src = gout + (uint64_t)r * (uint64_t)Z;
 #pragma unroll
                         for (int k = 0; k < KC; ++k) {
-                            if (colk[k] < L) v[u][k] = V::ldcs(src + colk[k]);
+                            if (colk[k] < L) v[u][k] = sign_by(V::ldcs(src + colk[k]), sb);
                             else
 #pragma unroll
                                 for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
@@ -408,7 +417,7 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                         const float* src = gout + (int64_t)row * d + j * Z;
 #pragma unroll
                         for (int k = 0; k < KC; ++k) {
-                            if (colk[k] < Lj) v[u][k] = V::ldcs(src + colk[k]);
+                            if (colk[k] < Lj) v[u][k] = sign_by(V::ldcs(src + colk[k]), sb);
                             else
 #pragma unroll
                                 for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
@@ -467,7 +476,7 @@ __global__ void __launch_bounds__(kThreads)
 k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     const unsigned long long* __restrict__ stats, int64_t npairs,
                     const float* __restrict__ gout, int d, int Z, int J, int log2J, int L,
-                    int64_t G, double* __restrict__ g) {
+                    int64_t G, uint32_t smask, double* __restrict__ g) {
     pdl_prologue();
     __shared__ unsigned long long s_ent[kWarps][kPiece];
     const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
@@ -504,7 +513,8 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
             for (int u = 0; u < kWU; ++u) {
                 const unsigned long long en = ent[b + u < (int)kPiece ? b + u : (int)kPiece - 1];
                 xs[u] = (b + u < n) ? (uint32_t)(en >> 32) : kBad;
-                const uint32_t r = (uint32_t)en;
+                const uint32_t r = (uint32_t)en & ~smask;
+                const uint32_t sb = (uint32_t)en & smask;
                 const float* src;
                 int Lj;
                 if (ZDIV) {
@@ -519,7 +529,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
                 for (int k = 0; k < KE; ++k) {
                     const int z = lane + 32 * k;
-                    v[u][k] = (xs[u] != kBad && z < Lj) ? __ldcs(src + z) : 0.f;
+                    v[u][k] = (xs[u] != kBad && z < Lj) ? sign_by(__ldcs(src + z), sb) : 0.f;
                 }
             }
             if (xs[kWU - 1] == cur) {
@@ -573,7 +583,8 @@ __device__ __forceinline__ void cp_async_wait() {
 __global__ void __launch_bounds__(kThreads)
 k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                const unsigned long long* __restrict__ stats, int64_t npairs,
-               const float* __restrict__ gout, int64_t G, double* __restrict__ g) {
+               const float* __restrict__ gout, int64_t G, uint32_t smask,
+               double* __restrict__ g) {
     pdl_prologue();
     __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
     __shared__ unsigned long long s_ent[kWarps][kAPiece];
@@ -607,7 +618,8 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                     const int part = pc & 7;
                     const int e = st * kAS + i;
                     if (e < n) {
-                        const uint32_t r = reinterpret_cast<const uint32_t*>(ent)[2 * e];  // low word
+                        const uint32_t r =
+                            reinterpret_cast<const uint32_t*>(ent)[2 * e] & ~smask;  // low word
                         cp_async16(&s_ring[warp][st % kAD][i][part * 4],
                                    gout + (uint64_t)r * 32u + (uint32_t)(part * 4));
                     }
@@ -634,6 +646,11 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
             float v[kAS];
 #pragma unroll
             for (int i = 0; i < kAS; ++i) v[i] = buf[i * 32 + lane];
+            if (smask) {
+                // signed hashing: each entry's sign is bit 31 of its low word
+#pragma unroll
+                for (int i = 0; i < kAS; ++i) v[i] = sign_by(v[i], ex[2 * i - 1] & smask);
+            }
             if (xlast == cur) {
                 const float a = (v[0] + v[1]) + (v[2] + v[3]);
                 const float b = (v[4] + v[5]) + (v[6] + v[7]);
@@ -668,7 +685,8 @@ cudaError_t warp_reduce_launch(const SortedBuffers& sb, int64_t npairs, const fl
     const int grid = grid_for(k_warp_range_reduce<KE, ZDIV, JPOW2>, sm_count,
                               (ntasks + kWarps - 1) / kWarps);
     return launch_k(k_warp_range_reduce<KE, ZDIV, JPOW2>, dim3(grid), dim3(kThreads), 0, st,
-                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g);
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask,
+                    g);
 }
 
 template <int KE>
@@ -692,7 +710,8 @@ cudaError_t reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* 
     const int64_t work_blocks = (ntasks + gpc - 1) / gpc;
     const int grid = grid_for(k_range_reduce<VW, KC, JPOW2, ZDIV>, sm_count, work_blocks, smem);
     return launch_k(k_range_reduce<VW, KC, JPOW2, ZDIV>, dim3(grid), dim3(kThreads), smem, st,
-                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, g, log2gs);
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g,
+                    log2gs);
 }
 
 template <int VW, int KC>
@@ -728,20 +747,26 @@ cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched
                     sb.bsum, sb.bnz, sb.start, tc);
 }
 
-cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, int sm_count,
-                                  cudaStream_t st) {
+cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
+                                  int sm_count, cudaStream_t st) {
     const int log2J = (J & (J - 1)) == 0 ? ceil_log2(J) : -1;
     const int64_t nseg = (npairs + kSeg - 1) / kSeg;
-    const int grid = grid_for(k_sort_scatter, sm_count, nseg);
-    return launch_k(k_sort_scatter, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs,
+    if (smask) {
+        const int grid = grid_for(k_sort_scatter<true>, sm_count, nseg);
+        return launch_k(k_sort_scatter<true>, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x,
+                        npairs, sb.q_row, J, log2J, sb.start, sb.cnt, sb.sorted_e);
+    }
+    const int grid = grid_for(k_sort_scatter<false>, sm_count, nseg);
+    return launch_k(k_sort_scatter<false>, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs,
                     sb.q_row, J, log2J, sb.start, sb.cnt, sb.sorted_e);
 }
 
-cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, int sm_count,
-                                cudaStream_t st) {
+cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
+                                int sm_count, cudaStream_t st) {
     const int64_t nseg = (npairs + kSeg - 1) / kSeg;
     const int grid = grid_for(k_sort_count, sm_count, nseg);
-    return launch_k(k_sort_count, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs, sb.cnt);
+    return launch_k(k_sort_count, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs, smask,
+                    sb.cnt);
 }
 
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
@@ -751,7 +776,7 @@ cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const 
         const int64_t ntasks = (npairs + kAPiece - 1) / kAPiece;   // upper bound
         const int grid = grid_for(k_async_reduce, sm_count, (ntasks + kWarps - 1) / kWarps);
         return launch_k(k_async_reduce, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e, sb.stats,
-                        npairs, gout, p.G, g);
+                        npairs, gout, p.G, p.smask, g);
     }
     // blocks of 32+ elements: one warp per task, one element per lane
     if (p.L >= 32) {

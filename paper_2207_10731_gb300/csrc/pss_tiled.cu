@@ -86,12 +86,25 @@ __device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t*
             const int j = k - qi * p.J;
             const int64_t q = qc0 + qi;
             const int64_t id = __ldg(idx + q);
-            if ((uint64_t)id < card) x = (XT)hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
-            else if (j == 0) record_bad_id(err, q);
+            if ((uint64_t)id < card) {
+                const uint64_t key = hash_key(p, (uint64_t)id, t, j);
+                x = (XT)hash_bucket(p, key) | (XT)hash_sign_bit(p, key);
+            } else if (j == 0) {
+                record_bad_id(err, q);
+            }
             s_x[k] = x;
         }
-        if (TOUCH) mark_touched_warp(tc, (uint64_t)x, x != Invalid<XT>::v, lane);
+        if (TOUCH)
+            mark_touched_warp(tc, (uint64_t)(x & ~(XT)p.smask), x != Invalid<XT>::v, lane);
     }
+}
+
+// One VW-wide load of a staged block (bucket x, column offset z); with signed
+// hashing (SG) the bucket carries the sign in bit 31, applied to the value.
+template <bool SG, typename V, typename XT>
+__device__ __forceinline__ typename V::T gather(const float* __restrict__ w, uint64_t G, XT x, int z) {
+    if (!SG) return V::ldg(w + G * (uint64_t)x + z);
+    return sign_by(V::ldg(w + G * (uint64_t)(x & ~(XT)0x80000000u) + z), (uint32_t)x & 0x80000000u);
 }
 
 // ---------------------------------------------------------------------------
@@ -103,7 +116,7 @@ constexpr int kWarpPairs = 512;   // staged pairs per warp and round
 
 // Hash the pairs [0, nq*J) of ids qc0.. into s_x (warp-cooperative); emits
 // the buckets for the sorted backward when asked.
-template <typename XT>
+template <typename XT, bool SG>
 __device__ __forceinline__ void warp_stage(const DevParams& p, const int64_t* __restrict__ idx,
                                            int t, uint64_t card, int64_t qc0, int nq, XT* s_x,
                                            DevError* err, uint32_t* __restrict__ pair_x,
@@ -119,8 +132,13 @@ __device__ __forceinline__ void warp_stage(const DevParams& p, const int64_t* __
             const int j = k - qi * p.J;
             const int64_t q = qc0 + qi;
             const int64_t id = __ldg(idx + q);
-            if ((uint64_t)id < card) x = (XT)hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
-            else if (j == 0) record_bad_id(err, q);
+            if ((uint64_t)id < card) {
+                const uint64_t key = hash_key(p, (uint64_t)id, t, j);
+                x = (XT)hash_bucket(p, key);
+                if (SG) x |= (XT)hash_sign_bit(p, key);
+            } else if (j == 0) {
+                record_bad_id(err, q);
+            }
             s_x[k] = x;
             if (pair_x) pair_x[qc0 * p.J + k] = (uint32_t)x;
         }
@@ -131,7 +149,7 @@ __device__ __forceinline__ void warp_stage(const DevParams& p, const int64_t* __
 // One-id tiles: stage by BAG.  s_x[bb*J + j] is the bucket of chunk j of the
 // id of bag bb (Invalid for an empty bag or a bad id), so the gather needs no
 // offsets; the id's output row is written here too.
-template <typename XT>
+template <typename XT, bool SG>
 __device__ __forceinline__ void warp_stage_bags(const DevParams& p, const int64_t* __restrict__ idx,
                                                 int t, uint64_t card, const int64_t* s_off, int nb,
                                                 XT* s_x, DevError* err,
@@ -150,8 +168,13 @@ __device__ __forceinline__ void warp_stage_bags(const DevParams& p, const int64_
             const int64_t q = s_off[bb];
             if (s_off[bb + 1] > q) {
                 const int64_t id = __ldg(idx + q);
-                if ((uint64_t)id < card) x = (XT)hash_bucket(p, hash_key(p, (uint64_t)id, t, j));
-                else if (j == 0) record_bad_id(err, q);
+                if ((uint64_t)id < card) {
+                    const uint64_t key = hash_key(p, (uint64_t)id, t, j);
+                    x = (XT)hash_bucket(p, key);
+                if (SG) x |= (XT)hash_sign_bit(p, key);
+                } else if (j == 0) {
+                    record_bad_id(err, q);
+                }
                 if (pair_x) pair_x[q * p.J + j] = (uint32_t)x;
                 if (q_row && j == 0) q_row[q] = row0 + (uint32_t)bb * (uint32_t)p.T;
             }
@@ -161,7 +184,7 @@ __device__ __forceinline__ void warp_stage_bags(const DevParams& p, const int64_
     __syncwarp();
 }
 
-template <int VW, int KC, typename XT>
+template <int VW, int KC, typename XT, bool SG>
 __global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
 k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                const int64_t* __restrict__ off, int64_t B, const float* __restrict__ w,
@@ -228,7 +251,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
 
         if (!multi && nb * J <= kWarpPairs) {
             // every bag holds at most one id: one load per bag, no accumulation
-            warp_stage_bags<XT>(p, idx, t, card, s_off, nb, s_x, err, pair_x, q_row,
+            warp_stage_bags<XT, SG>(p, idx, t, card, s_off, nb, s_x, err, pair_x, q_row,
                                 (uint32_t)(b0 * p.T + t), lane);
             float* orow0 = obase + gb0 * ostride;
             for (int bb0 = gb0; bb0 < gb1; bb0 += kU) {
@@ -242,7 +265,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                         for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
                         if (bb < gb1 && col.v[k]) {
                             const XT x = s_x[bb * J + col.j[k]];
-                            if (x != Invalid<XT>::v) v[u][k] = V::ldg(w + G * (uint64_t)x + col.z[k]);
+                            if (x != Invalid<XT>::v) v[u][k] = gather<SG, V>(w, G, x, col.z[k]);
                         }
                     }
                 }
@@ -278,7 +301,8 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                 if (q >= sw1) {
                     sw0 = q;
                     sw1 = (qb - q) < qcw ? qb : q + qcw;
-                    warp_stage<XT>(p, idx, t, card, sw0, (int)(sw1 - sw0), s_x, err, pair_x, lane);
+                    warp_stage<XT, SG>(p, idx, t, card, sw0, (int)(sw1 - sw0), s_x, err, pair_x,
+                                       lane);
                 }
                 const int64_t qend = c < sw1 ? c : sw1;
                 for (int64_t qs = q; qs < qend; qs += (int64_t)kU * ng) {
@@ -292,7 +316,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                             for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
                             if (qq < qend && col.v[k]) {
                                 const XT x = s_x[(int)(qq - sw0) * J + col.j[k]];
-                                if (x != Invalid<XT>::v) v[u][k] = V::ldg(w + G * (uint64_t)x + col.z[k]);
+                                if (x != Invalid<XT>::v) v[u][k] = gather<SG, V>(w, G, x, col.z[k]);
                             }
                         }
                         if (qq < qend && q_row && lg == 0) q_row[qq] = row;
@@ -427,7 +451,8 @@ k_scatter_tiled(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                         if (!col.v[k]) continue;
                         const XT x = s_x[(int)(q + u - qc0) * J + col.j[k]];
                         if (x != Invalid<XT>::v)
-                            Acc<VW, AT>::red(target + G * (uint64_t)x + col.z[k], row[k]);
+                            Acc<VW, AT>::red(target + G * (uint64_t)(x & ~(XT)p.smask) + col.z[k],
+                                             sign_by(row[k], (uint32_t)x & p.smask));
                     }
                 }
             }
@@ -452,7 +477,7 @@ size_t tile_smem(const TileGeom& g, const DevParams& p, size_t xbytes) {
     return sizeof(int64_t) * (size_t)(g.tb + 1) + xbytes * (size_t)g.qc * (size_t)p.J;
 }
 
-template <int VW, int KC, typename XT>
+template <int VW, int KC, typename XT, bool SG>
 cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                      const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
                      uint32_t* pair_x, uint32_t* q_row, int sm_count,
@@ -463,9 +488,9 @@ cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* id
                                           (size_t)kWarpPairs * sizeof(XT));
     const int64_t ntiles = (int64_t)p.T * tpt;
     if (ntiles >= ((int64_t)1 << 31)) return cudaErrorInvalidValue;
-    const int grid = grid_for(k_forward_warp<VW, KC, XT>, sm_count, (ntiles + kWarps - 1) / kWarps,
+    const int grid = grid_for(k_forward_warp<VW, KC, XT, SG>, sm_count, (ntiles + kWarps - 1) / kWarps,
                               smem);
-    return launch_k(k_forward_warp<VW, KC, XT>, dim3(grid), dim3(kThreads), smem, st, p, idx, nnz,
+    return launch_k(k_forward_warp<VW, KC, XT, SG>, dim3(grid), dim3(kThreads), smem, st, p, idx, nnz,
                     off, B, w, out, err, pair_x, q_row, lay.log2gs, wb, tpt);
 }
 
@@ -487,10 +512,13 @@ cudaError_t fwd_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, 
                   uint32_t* pair_x, uint32_t* q_row, int sm_count,
                   cudaStream_t st) {
     if (p.R < 0xffffffffull)
-        return fwd_inst<VW, KC, uint32_t>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row,
-                                          sm_count, st);
-    return fwd_inst<VW, KC, uint64_t>(p, lay, idx, nnz, off, B, w, out, err, nullptr, nullptr,
-                                      sm_count, st);
+        return p.smask ? fwd_inst<VW, KC, uint32_t, true>(p, lay, idx, nnz, off, B, w, out, err,
+                                                           pair_x, q_row, sm_count, st)
+                       : fwd_inst<VW, KC, uint32_t, false>(p, lay, idx, nnz, off, B, w, out, err,
+                                                            pair_x, q_row, sm_count, st);
+    // R >= 2^32: 64-bit buckets, never signed (signed hashing needs R < 2^31)
+    return fwd_inst<VW, KC, uint64_t, false>(p, lay, idx, nnz, off, B, w, out, err, nullptr,
+                                             nullptr, sm_count, st);
 }
 
 template <int VW, int KC, typename AT>

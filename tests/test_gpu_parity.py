@@ -425,6 +425,91 @@ def test_compression_sweep(logM):
 
 
 # --------------------------------------------------------------------------
+# signed hashing (NEXT row: a +-1 per (id, chunk) from a second hash)
+SIGNED_CASES = [
+    dict(name="tiny"),
+    dict(name="kaggle"),
+    dict(name="tb", B=4096),
+    dict(name="multihot", B=1024),
+    dict(name="multihot", B=777, bag=("uniform", 0, 6)),      # empty bags, ragged tail
+    dict(name="tiny", Z=1, G=1),                              # scalar kernels
+    dict(name="kaggle", Z=3, G=2, B=300),                     # Z does not divide d
+    dict(name="tb", B=500, d=200, Z=32),                      # two columns per lane
+]
+
+
+def _signed_pair(w, path):
+    from oracle import OraclePSS
+    h, o_u = gu.make_pair(w)
+    o = OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, signed=True)
+    h.set_option(binding.OPT_SIGNED, 1)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    return h, o, o_u
+
+
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("case", SIGNED_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_signed_hashing_forward_and_grad_parity(case, path):
+    w = _wl(case)
+    h, o, o_u = _signed_pair(w, path)
+    assert h.info()["signed_hash"] == 1
+    assert (h.info()["A2"], h.info()["B2"]) == (o.A2, o.B2)
+    out = gu.host(h.forward(*_batch_cuda(w), w.B)).ravel()
+    ref, bad = o.forward(w.w0, w.indices, w.offsets, w.B)
+    assert bad == -1
+    # |s * w| = |w|: the unsigned oracle gives the conditioning bounds
+    gu.check_forward(out, ref, _abs_pool(o_u, w.w0, w), what="signed forward")
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    gref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
+    A = o_u.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g, gref, A, what="signed grad")
+    assert h.info()["last_path"] == PATHS[path]
+    h.close()
+
+
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("opt", ["sgd", "adagrad"])
+def test_signed_hashing_step_dyadic_bit_exact(opt, path):
+    # dyadic inputs: every sum is exact, so the signed step must give the
+    # oracle's bits on both paths
+    w = wl.make_workload("kaggle", B=1024, grad="dyadic", w0="dyadic", opt=opt)
+    w.lr = 0.125
+    h, o, _ = _signed_pair(w, path)
+    h.forward(*_batch_cuda(w), w.B)
+    out = gu.host(h.forward(*_batch_cuda(w), w.B)).ravel()
+    ref, _ = o.forward(w.w0, w.indices, w.offsets, w.B)
+    np.testing.assert_array_equal(out, ref)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    wg, Gg = h.get_state()
+    w2, G2, _ = o.step(w.w0, np.zeros(w.M, np.float32), w.indices, w.offsets, w.B, w.grad_out,
+                       opt, w.lr, w.eps)
+    np.testing.assert_array_equal(gu.host(wg), w2)
+    if opt == "adagrad":
+        np.testing.assert_array_equal(gu.host(Gg), G2)
+    h.close()
+
+
+def test_signed_option_forgets_the_batch_and_needs_small_R():
+    w = wl.make_workload("tiny")
+    h, _ = gu.make_pair(w)
+    h.forward(*_batch_cuda(w), w.B)
+    h.set_option(binding.OPT_SIGNED, 1)
+    with pytest.raises(binding.PSSError) as e:
+        h.backward_update(gu.cuda(w.grad_out), w.lr)
+    assert e.value.status == binding.PSS_ERR_STATE
+    assert h.get_option(binding.OPT_SIGNED) == 1
+    with pytest.raises(binding.PSSError):
+        h.set_option(binding.OPT_SIGNED, 2)
+    h.close()
+    # R >= 2^31 block starts: the sign cannot travel in bit 31
+    big = binding.PSS(w.cards, dim=16, M=(1 << 31) + 64, Z=16, G=1, seed=0, optimizer="sgd")
+    with pytest.raises(binding.PSSError) as e:
+        big.set_option(binding.OPT_SIGNED, 1)
+    assert e.value.status == binding.PSS_ERR_UNSUPPORTED
+    big.close()
+
+
+# --------------------------------------------------------------------------
 # host buffers through the same C-ABI calls (the end-to-end path)
 def test_host_buffers_match_device_buffers():
     # dyadic inputs: every sum is exact, so both paths must give the same bits
