@@ -179,10 +179,10 @@ def _oracle_sample(w: wl.Workload, rows: int):
 
 
 def _oracle_rate(w: wl.Workload, budget_s: float, forward_only: bool = False,
-                 max_rows: int = None):
+                 max_rows: int = None, signed: bool = False):
     """Time the CPU oracle (as it stands) on bounded samples of the workload."""
     import oracle
-    o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed)
+    o = oracle.OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, signed=signed)
     wcur = w.w0.copy() if w.w0 is not None else None
     Gcur = np.zeros(w.M, np.float32)
     rows = min(w.B, max_rows or 256)
@@ -432,7 +432,8 @@ def run_gpu(args):
         step_gbs = step_bytes / (elapsed_ms / args.steps / 1e3) / 1e9 * world
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
-            rate, rows, reps, nnz_s, tot = _oracle_rate(w, args.cpu_budget, args.forward_only)
+            rate, rows, reps, nnz_s, tot = _oracle_rate(w, args.cpu_budget, args.forward_only,
+                                                        signed=args.signed)
             cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                    "sample": (f"first {rows} of {w.B} batch rows x {w.T} tables "
                               f"({nnz_s} lookups) per step, {reps} steps, {tot:.1f} s: "
