@@ -47,7 +47,7 @@ class _Pss(ctypes.Structure):
                 ("Z", ctypes.c_int64), ("G", ctypes.c_int64), ("J", ctypes.c_int64),
                 ("L", ctypes.c_int64), ("R", ctypes.c_int64), ("A", ctypes.c_uint64),
                 ("B0", ctypes.c_uint64), ("cards", ctypes.c_void_p), ("sgn", ctypes.c_int64),
-                ("A2", ctypes.c_uint64), ("B2", ctypes.c_uint64)]
+                ("A2", ctypes.c_uint64), ("B2", ctypes.c_uint64), ("circ", ctypes.c_int64)]
 
 
 def _load():
@@ -61,6 +61,7 @@ def _load():
                 "oracle_hash_params": (None, [u64, vp, vp]),
                 "oracle_sign_params": (None, [u64, vp, vp]),
                 "oracle_set_signed": (None, [vp, i64]),
+                "oracle_set_circular": (ctypes.c_int, [vp, i64]),
                 "oracle_sign": (i64, [vp, i64, i64, i64]),
                 "oracle_signs": (ctypes.c_int, [vp, vp, i64, vp, i64, vp]),
                 "oracle_init": (ctypes.c_int, [vp, vp, i64, i64, i64, i64, i64, u64]),
@@ -117,7 +118,7 @@ class OraclePSS:
     block-start alignment G, hash seed.  All arrays are numpy, host memory."""
 
     def __init__(self, cards, d: int, M: int, Z: int, G: int = 4, seed: int = 0,
-                 signed: bool = False):
+                 signed: bool = False, circular: bool = False):
         self._lib = _load()
         self.cards = _c(cards, np.int64)
         self.T = int(self.cards.shape[0])
@@ -132,6 +133,12 @@ class OraclePSS:
         self.A2, self.B2 = int(self._p.A2), int(self._p.B2)
         self.signed = bool(signed)
         self._lib.oracle_set_signed(ctypes.byref(self._p), 1 if signed else 0)
+        self.circular = bool(circular)
+        if circular:
+            rc = self._lib.oracle_set_circular(ctypes.byref(self._p), 1)
+            if rc != 0:
+                raise OracleError(f"oracle_set_circular failed ({rc})")
+            self.R = int(self._p.R)
 
     def _pp(self):
         return ctypes.byref(self._p)

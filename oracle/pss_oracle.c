@@ -40,7 +40,11 @@
  *     also gets a sign s = +-1 from a second hash of the same family with its
  *     own parameters A2 = 1 + (s3 mod (P-1)), B2 = s4 mod P (the third and
  *     fourth splitmix64 outputs): s = -1 when (A2*key + B2) mod P is odd.  The
- *     forward adds s * block, the backward adds s * upstream gradient.
+ *     forward adds s * block, the backward adds s * upstream gradient;
+ *   - circular array (optional; the other reading of the printed range
+ *     {0..|M_r|}): R = M / G block starts (G must divide M), and element z of
+ *     the block at loc is M[(loc + z) mod M], so blocks near the end wrap to
+ *     the start of the array.
  */
 #include <stdint.h>
 #include <stdlib.h>
@@ -56,6 +60,7 @@ typedef struct {
     const int64_t* cards;         /* host, T cardinalities (not owned) */
     int64_t sgn;                  /* 1: signed hashing */
     uint64_t A2, B2;              /* sign-hash parameters */
+    int64_t circ;                 /* 1: circular array */
 } oracle_pss;
 
 /* splitmix64 (Steele, Lea & Flood, "Fast splittable pseudorandom number
@@ -124,7 +129,30 @@ int oracle_init(oracle_pss* p, const int64_t* cards, int64_t T, int64_t d, int64
     oracle_hash_params(seed, &p->A, &p->B0);
     oracle_sign_params(seed, &p->A2, &p->B2);
     p->sgn = 0;
+    p->circ = 0;
     return 0;
+}
+
+/* Turn the circular array on (1) or off (0).  On: R = M / G block starts
+ * (G must divide M; returns -5 otherwise and leaves the instance unchanged). */
+int oracle_set_circular(oracle_pss* p, int64_t on)
+{
+    if (on) {
+        if (p->M % p->G) return -5;
+        p->R = p->M / p->G;
+        p->circ = 1;
+    } else {
+        p->R = (p->M - p->L) / p->G + 1;
+        p->circ = 0;
+    }
+    return 0;
+}
+
+/* Element of the shared array that holds offset z of the block at loc. */
+static int64_t elem(const oracle_pss* p, int64_t loc, int64_t z)
+{
+    int64_t e = loc + z;
+    return (p->circ && e >= p->M) ? e - p->M : e;
 }
 
 /* Turn signed hashing on (1) or off (0). */
@@ -237,7 +265,7 @@ int oracle_pool(const oracle_pss* p, const float* w, const int64_t* locs, int64_
                     int64_t Lj = d - j * p->Z < p->Z ? d - j * p->Z : p->Z;
                     double sg = signs ? (double)signs[q * p->J + j] : 1.0;
                     if (loc < 0) continue;
-                    for (int64_t z = 0; z < Lj; ++z) acc[j * p->Z + z] += sg * (double)w[loc + z];
+                    for (int64_t z = 0; z < Lj; ++z) acc[j * p->Z + z] += sg * (double)w[elem(p, loc, z)];
                 }
             for (int64_t k = 0; k < d; ++k) out[(b * T + t) * d + k] = (float)acc[k];
         }
@@ -288,7 +316,7 @@ int oracle_scatter(const oracle_pss* p, const int64_t* locs, int64_t nnz, const 
                     int64_t Lj = d - j * p->Z < p->Z ? d - j * p->Z : p->Z;
                     double sg = signs ? (double)signs[q * p->J + j] : 1.0;
                     if (loc < 0) continue;
-                    for (int64_t z = 0; z < Lj; ++z) g[loc + z] += sg * (double)go[j * p->Z + z];
+                    for (int64_t z = 0; z < Lj; ++z) g[elem(p, loc, z)] += sg * (double)go[j * p->Z + z];
                 }
         }
     return 0;
@@ -348,6 +376,15 @@ int oracle_grad_at(const oracle_pss* p, const int64_t* indices, int64_t nnz, con
                     int64_t loc = oracle_location(p, id, t, j);
                     int64_t Lj = d - j * p->Z < p->Z ? d - j * p->Z : p->Z;
                     double sg = (double)oracle_sign(p, id, t, j);
+                    if (p->circ && loc + Lj > p->M) {
+                        /* a block that wraps: look every element up */
+                        for (int64_t z = 0; z < Lj; ++z) {
+                            int64_t e = elem(p, loc, z);
+                            int64_t k = lower_bound_i64(elems, n_elems, e);
+                            if (k < n_elems && elems[k] == e) g_at[k] += sg * (double)go[j * p->Z + z];
+                        }
+                        continue;
+                    }
                     for (int64_t k = lower_bound_i64(elems, n_elems, loc);
                          k < n_elems && elems[k] < loc + Lj; ++k)
                         g_at[k] += sg * (double)go[j * p->Z + (elems[k] - loc)];

@@ -235,6 +235,66 @@ def test_signed_grad_at_matches_signed_dense_grad():
     np.testing.assert_array_equal(o.grad_at(idx, off, 6, go, elems), g[elems])
 
 
+# --------------------------------------------------------------------------
+# circular array (the other reading of the printed range {0..|M_r|}): R = M/G
+# starts, and blocks near the end of M wrap to its start
+@pytest.mark.parametrize("Z,G,d,signed", [(16, 4, 16, False), (4, 2, 16, False), (32, 4, 16, True),
+                                          (3, 1, 10, False)])
+def test_circular_forward_and_grad_equal_wrapping_bruteforce_matrix(Z, G, d, signed):
+    T, B, M = 2, 4, 64          # small M: many blocks wrap
+    wrapped = 0
+    for seed in range(4):
+        cards, idx, off, w, go = _tiny_case(seed, T=T, B=B, d=d, M=M, Z=Z, G=G, max_bag=4)
+        o = OraclePSS(cards, d=d, M=M, Z=Z, G=G, seed=seed, signed=signed, circular=True)
+        A, B0 = bh.params(seed)
+        A2, B2 = bh.sign_params(seed)
+        L, J = min(Z, d), -(-d // Z)
+        R = M // G
+        assert o.R == R
+        rows, cols, vals = [], [], []
+        for t in range(T):
+            for b in range(B):
+                s = t * B + b
+                for q in range(off[s], off[s + 1]):
+                    i = int(idx[q])
+                    for k in range(d):
+                        j, z = divmod(k, Z)
+                        loc = bh.location(A, B0, R, G, T, J, i, t, j)
+                        wrapped += (loc + z) >= M
+                        rows.append((b * T + t) * d + k)
+                        cols.append((loc + z) % M)
+                        vals.append(bh.sign(A2, B2, T, J, i, t, j) if signed else 1)
+        P = sp.coo_matrix((vals, (rows, cols)), shape=(B * T * d, M)).tocsr()
+        out, bad = o.forward(w, idx, off, B)
+        assert bad == -1
+        np.testing.assert_array_equal(out, (P @ w.astype(np.float64)).astype(np.float32))
+        np.testing.assert_array_equal(o.grad(idx, off, B, go), P.T @ go.astype(np.float64))
+    assert wrapped > 0
+
+
+def test_circular_with_block_aligned_starts_is_the_plain_mapping():
+    # G = L: R = M/L starts either way and no block crosses the end, so the two
+    # readings of the range coincide
+    cards, idx, off, w, go = _tiny_case(3, T=3, B=8, d=32, M=512, Z=16, G=16, max_bag=5)
+    a = OraclePSS(cards, d=32, M=512, Z=16, G=16, seed=2, circular=True)
+    b = OraclePSS(cards, d=32, M=512, Z=16, G=16, seed=2)
+    assert a.R == b.R
+    np.testing.assert_array_equal(a.forward(w, idx, off, 8)[0], b.forward(w, idx, off, 8)[0])
+    np.testing.assert_array_equal(a.grad(idx, off, 8, go), b.grad(idx, off, 8, go))
+
+
+def test_circular_adjoint_sparse_gradient_and_rejection():
+    cards, idx, off, w, go = _tiny_case(6, T=3, B=8, d=16, M=96, Z=8, G=4, max_bag=5)
+    o = OraclePSS(cards, d=16, M=96, Z=8, G=4, seed=4, circular=True, signed=True)
+    out, _ = o.forward(w, idx, off, 8)
+    g = o.grad(idx, off, 8, go)
+    assert float(np.dot(out.astype(np.float64), go.astype(np.float64))) == float(np.dot(w.astype(np.float64), g))
+    elems = np.flatnonzero(g)
+    np.testing.assert_array_equal(o.grad_at(idx, off, 8, go, elems), g[elems])
+    with pytest.raises(OracleError):
+        OraclePSS(cards, d=16, M=98, Z=8, G=4, seed=4, circular=True)
+
+
 def test_forward_bruteforce_non_dyadic():
     cards, idx, off, w, go = _tiny_case(5, T=3, B=8, d=16, M=300, Z=4, G=1, max_bag=6, dy=False)
     o = OraclePSS(cards, d=16, M=300, Z=4, G=1, seed=9)
