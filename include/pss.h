@@ -115,7 +115,15 @@ typedef enum {
      * last forward's batch (the next backward needs a new forward).
      * pss_compute_locations returns locations only; pss_grad_noalloc is
      * unsigned. */
-    PSS_OPT_SIGNED = 6
+    PSS_OPT_SIGNED = 6,
+    /* 1: circular array, the other reading of the printed range of h
+     * (Sec. 2.5): R = M / G block starts, and element z of the block at loc is
+     * M[(loc + z) mod M], so blocks near the end wrap to the start of M.
+     * Needs G to divide M (PSS_ERR_UNSUPPORTED otherwise).  The optimizer pass
+     * is then always the dense one.  Changing it synchronises the device,
+     * changes R (pss_get_info) and forgets the last forward's batch.
+     * pss_grad_noalloc does not wrap. */
+    PSS_OPT_CIRCULAR = 7
 } pss_option;
 
 
@@ -147,6 +155,7 @@ typedef struct {
     double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass, or -1 */
     uint64_t A2, B2;           /* sign-hash parameters derived from the seed */
     int64_t signed_hash;       /* PSS_OPT_SIGNED */
+    int64_t circular;          /* PSS_OPT_CIRCULAR */
 } pss_info;
 
 /*

@@ -24,6 +24,7 @@ PSS_OK, PSS_ERR_INVALID_ARG, PSS_ERR_OOM, PSS_ERR_CUDA, PSS_ERR_STATE, PSS_ERR_I
 PSS_SGD, PSS_ADAGRAD = 0, 1
 OPT_BACKWARD_PATH, OPT_UPDATE_MODE, OPT_PROFILE, OPT_SYNC_CHECK, OPT_ACCUM = 1, 2, 3, 4, 5
 OPT_SIGNED = 6
+OPT_CIRCULAR = 7
 ACCUM_F64, ACCUM_F32 = 0, 1
 PATH_AUTO, PATH_ATOMIC, PATH_SORTED = 0, 1, 2
 UPDATE_AUTO, UPDATE_DENSE, UPDATE_TOUCHED = 0, 1, 2
@@ -47,7 +48,8 @@ class PSSInfo(ctypes.Structure):
                 ("B0", ctypes.c_uint64), ("optimizer", ctypes.c_int64),
                 ("kernel_launches", ctypes.c_int64), ("last_path", ctypes.c_int64),
                 ("last_collision_rate", ctypes.c_double), ("A2", ctypes.c_uint64),
-                ("B2", ctypes.c_uint64), ("signed_hash", ctypes.c_int64)]
+                ("B2", ctypes.c_uint64), ("signed_hash", ctypes.c_int64),
+                ("circular", ctypes.c_int64)]
 
 
 class PSSError(RuntimeError):

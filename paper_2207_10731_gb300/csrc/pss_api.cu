@@ -88,6 +88,11 @@ struct pss_handle {
     cudaStream_t s_h2d = nullptr;
     cudaEvent_t ev_grad_ready = nullptr, ev_grad_free = nullptr, ev_alloc = nullptr;
     bool grad_free_pending = false;
+    // circular array: R = M/G starts, blocks past M wrap to its start.  w and
+    // the gradient accumulators have L extra elements past M: w's mirror
+    // M[0 .. L) (refreshed after every write of w), the accumulators' collect
+    // the wrapped contributions until they are folded into the head.
+    bool circ = false;
     bool stats_pending = false;
 
     // profiling
@@ -251,13 +256,50 @@ pss_status check_error_word(pss_handle* h, cudaStream_t st, int64_t* first_bad) 
 pss_status ensure_grad(pss_handle* h, cudaStream_t st) {
     if (h->accum == PSS_ACCUM_F32) {
         if (h->g) return PSS_OK;
-        PSS_TRY(cudaMalloc(&h->g, sizeof(float) * (size_t)h->dp.M));
-        PSS_TRY(cudaMemsetAsync(h->g, 0, sizeof(float) * (size_t)h->dp.M, st));
+        PSS_TRY(cudaMalloc(&h->g, sizeof(float) * (size_t)(h->dp.M + h->dp.L)));
+        PSS_TRY(cudaMemsetAsync(h->g, 0, sizeof(float) * (size_t)(h->dp.M + h->dp.L), st));
         return PSS_OK;
     }
     if (h->g64) return PSS_OK;
-    PSS_TRY(cudaMalloc(&h->g64, sizeof(double) * (size_t)h->dp.M));
-    PSS_TRY(cudaMemsetAsync(h->g64, 0, sizeof(double) * (size_t)h->dp.M, st));
+    PSS_TRY(cudaMalloc(&h->g64, sizeof(double) * (size_t)(h->dp.M + h->dp.L)));
+    PSS_TRY(cudaMemsetAsync(h->g64, 0, sizeof(double) * (size_t)(h->dp.M + h->dp.L), st));
+    return PSS_OK;
+}
+
+// Buffers sized by the number of block starts R, released when R changes (they
+// are allocated again on first use).  The caller has synchronised the device.
+void release_r_buffers(pss_handle* h) {
+    for (void* b : {(void*)h->sb.cnt, (void*)h->sb.start, (void*)h->sb.bsum, (void*)h->sb.bnz,
+                    (void*)h->sb.stats, (void*)h->touched.bitmap, (void*)h->touched.list,
+                    (void*)h->touched.count})
+        if (b) cudaFree(b);
+    if (h->stats_host) cudaFreeHost(h->stats_host);
+    if (h->stats_ev) cudaEventDestroy(h->stats_ev);
+    h->sb.cnt = h->sb.start = h->sb.bsum = h->sb.bnz = nullptr;
+    h->sb.stats = nullptr;
+    h->stats_host = nullptr;
+    h->stats_ev = nullptr;
+    h->stats_pending = false;
+    h->sb_counters = false;
+    h->touched = Touched{};
+    h->touched_words = 0;
+}
+
+// Circular array: refresh w's mirror of M[0 .. L) after a write of w.
+pss_status mirror_head(pss_handle* h, cudaStream_t st) {
+    if (h->circ)
+        PSS_TRY(cudaMemcpyAsync(h->w + h->dp.M, h->w, sizeof(float) * (size_t)h->dp.L,
+                                cudaMemcpyDeviceToDevice, st));
+    return PSS_OK;
+}
+
+// Circular array: fold the accumulator's wrapped contributions into its head.
+pss_status fold_tail(pss_handle* h, bool f64, cudaStream_t st) {
+    if (h->circ) {
+        LaunchScope ls(h, PSS_K_MISC, st);
+        PSS_TRY(launch_fold_tail(f64 ? h->g64 : nullptr, f64 ? nullptr : h->g, (int64_t)h->dp.M,
+                                 h->dp.L, st));
+    }
     return PSS_OK;
 }
 
@@ -284,6 +326,7 @@ pss_status ensure_touched(pss_handle* h, int64_t pairs, cudaStream_t st) {
 }
 
 bool use_touched(const pss_handle* h, int64_t pairs) {
+    if (h->circ) return false;   // the ownership rule of the touched pass does not wrap
     if (h->update_mode == PSS_UPDATE_DENSE) return false;
     if (h->update_mode == PSS_UPDATE_TOUCHED) return true;
     // the dense pass touches every element of M once; the touched pass visits
@@ -468,8 +511,10 @@ pss_status pss_create(const int64_t* cards, int32_t T, int32_t dim, int64_t M, i
 
     pss_status rc = PSS_OK;
     do {
-        if ((rc = cuda_status(cudaMalloc(&h->w, sizeof(float) * (size_t)M))) != PSS_OK) break;
-        if ((rc = cuda_status(cudaMemsetAsync(h->w, 0, sizeof(float) * (size_t)M, st))) != PSS_OK) break;
+        // L elements past M: the circular array's mirror of M[0 .. L)
+        if ((rc = cuda_status(cudaMalloc(&h->w, sizeof(float) * (size_t)(M + L)))) != PSS_OK) break;
+        if ((rc = cuda_status(cudaMemsetAsync(h->w, 0, sizeof(float) * (size_t)(M + L), st))) != PSS_OK)
+            break;
         if (opt == PSS_ADAGRAD) {
             if ((rc = cuda_status(cudaMalloc(&h->Gacc, sizeof(float) * (size_t)M))) != PSS_OK) break;
             if ((rc = cuda_status(cudaMemsetAsync(h->Gacc, 0, sizeof(float) * (size_t)M, st))) != PSS_OK) break;
@@ -534,7 +579,7 @@ pss_status pss_set_weights(pss_handle* h, const float* w, int64_t n, pss_stream 
     DeviceGuard g(h->device);
     PSS_TRY(cudaMemcpyAsync(h->w, w, sizeof(float) * (size_t)n, cudaMemcpyDefault,
                             reinterpret_cast<cudaStream_t>(stream)));
-    return PSS_OK;
+    return mirror_head(h, reinterpret_cast<cudaStream_t>(stream));
 }
 
 pss_status pss_get_weights(pss_handle* h, float* w, int64_t n, pss_stream stream) {
@@ -563,7 +608,7 @@ pss_status pss_set_state(pss_handle* h, const float* w, const float* G, int64_t 
     PSS_TRY(cudaMemcpyAsync(h->w, w, sizeof(float) * (size_t)n, cudaMemcpyDefault, st));
     if (h->opt == PSS_ADAGRAD)
         PSS_TRY(cudaMemcpyAsync(h->Gacc, G, sizeof(float) * (size_t)n, cudaMemcpyDefault, st));
-    return PSS_OK;
+    return mirror_head(h, st);
 }
 
 pss_status pss_compute_locations(pss_handle* h, const int64_t* indices, int64_t nnz,
@@ -712,6 +757,7 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
         if (touch && (rc = ensure_touched(h, pairs, st)) != PSS_OK) return rc;
         if ((rc = sorted_into64(h, dg, staged, touch, st)) != PSS_OK) return rc;
         if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
+        if ((rc = fold_tail(h, true, st)) != PSS_OK) return rc;
         {
             LaunchScope ls(h, PSS_K_UPDATE, st);
             if (touch)
@@ -725,7 +771,7 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
             LaunchScope ls(h, PSS_K_MISC, st);
             PSS_TRY(launch_touched_clear(h->touched, h->sm_count, st));
         }
-    } else if (h->accum == PSS_ACCUM_F32 && !ada) {
+    } else if (h->accum == PSS_ACCUM_F32 && !ada && !h->circ) {
         // SGD is linear in g: scatter -lr * grad_out straight into M.
         if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
         if (lr != 0.f && (rc = scatter_into(h, dg, -lr, h->w, false, st)) != PSS_OK) return rc;
@@ -741,6 +787,7 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
             rc = scatter_into64(h, dg, touch, st);
         if (rc != PSS_OK) return rc;
         if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
+        if ((rc = fold_tail(h, h->accum != PSS_ACCUM_F32, st)) != PSS_OK) return rc;
         {
             LaunchScope ls(h, PSS_K_UPDATE, st);
             if (h->accum == PSS_ACCUM_F32) {
@@ -764,6 +811,7 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
             PSS_TRY(launch_touched_clear(h->touched, h->sm_count, st));
         }
     }
+    if ((rc = mirror_head(h, st)) != PSS_OK) return rc;
     if (h->sync_check) return check_error_word(h, st, nullptr);
     return PSS_OK;
 }
@@ -790,18 +838,26 @@ pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, 
         if (rc != PSS_OK) return rc;
         if ((rc = sorted_into64(h, dg, staged, false, st)) != PSS_OK) return rc;
         if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
+        if ((rc = fold_tail(h, true, st)) != PSS_OK) return rc;
         LaunchScope ls(h, PSS_K_MISC, st);
         PSS_TRY(launch_grad_export(h->g64, grad, h->dp.M, h->sm_count, st));
-    } else if (h->accum == PSS_ACCUM_F32) {
+    } else if (h->accum == PSS_ACCUM_F32 && !h->circ) {
         PSS_TRY(cudaMemsetAsync(grad, 0, sizeof(float) * (size_t)h->dp.M, st));
         if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
         if ((rc = scatter_into(h, dg, 1.0f, grad, false, st)) != PSS_OK) return rc;
         if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
     } else {
-        if ((rc = ensure_grad(h, st)) != PSS_OK) return rc;
+        // (the circular array always takes the fp64 accumulator here: the
+        // caller's grad has no room for the wrapped tail)
+        const int64_t saved = h->accum;
+        h->accum = PSS_ACCUM_F64;
+        rc = ensure_grad(h, st);
+        h->accum = saved;
+        if (rc != PSS_OK) return rc;
         if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
         if ((rc = scatter_into64(h, dg, false, st)) != PSS_OK) return rc;
         if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
+        if ((rc = fold_tail(h, true, st)) != PSS_OK) return rc;
         LaunchScope ls(h, PSS_K_MISC, st);
         PSS_TRY(launch_grad_export(h->g64, grad, h->dp.M, h->sm_count, st));
     }
@@ -832,6 +888,24 @@ pss_status pss_set_option(pss_handle* h, int32_t key, int64_t value) {
             if (value != PSS_ACCUM_F64 && value != PSS_ACCUM_F32) return PSS_ERR_INVALID_ARG;
             h->accum = value;
             return PSS_OK;
+        case PSS_OPT_CIRCULAR: {
+            if (value != 0 && value != 1) return PSS_ERR_INVALID_ARG;
+            const int64_t M = h->dp.M, G = h->dp.G, L = h->dp.L;
+            if (value && M % G) return PSS_ERR_UNSUPPORTED;
+            const uint64_t R = value ? (uint64_t)(M / G) : (uint64_t)((M - L) / G + 1);
+            if (h->dp.smask && R >= (uint64_t(1) << 31)) return PSS_ERR_UNSUPPORTED;
+            if ((value != 0) == h->circ) return PSS_OK;
+            DeviceGuard g(h->device);
+            PSS_TRY(cudaDeviceSynchronize());
+            release_r_buffers(h);
+            h->dp.R = R;
+            h->dp.Rinv = UINT64_MAX / R;
+            h->circ = value != 0;
+            h->have_batch = false;
+            if (h->circ)
+                PSS_TRY(cudaMemcpy(h->w + M, h->w, sizeof(float) * (size_t)L, cudaMemcpyDeviceToDevice));
+            return PSS_OK;
+        }
         case PSS_OPT_SIGNED: {
             if (value != 0 && value != 1) return PSS_ERR_INVALID_ARG;
             // the sign travels in bit 31 of a 32-bit bucket index
@@ -854,6 +928,7 @@ pss_status pss_get_option(pss_handle* h, int32_t key, int64_t* value) {
         case PSS_OPT_SYNC_CHECK: *value = h->sync_check; return PSS_OK;
         case PSS_OPT_ACCUM: *value = h->accum; return PSS_OK;
         case PSS_OPT_SIGNED: *value = h->dp.smask ? 1 : 0; return PSS_OK;
+        case PSS_OPT_CIRCULAR: *value = h->circ ? 1 : 0; return PSS_OK;
     }
     return PSS_ERR_INVALID_ARG;
 }
@@ -880,6 +955,7 @@ pss_status pss_get_info(pss_handle* h, pss_info* info) {
     info->A2 = h->dp.A2;
     info->B2 = h->dp.B2;
     info->signed_hash = h->dp.smask ? 1 : 0;
+    info->circular = h->circ ? 1 : 0;
     info->optimizer = h->opt;
     info->kernel_launches = h->launches;
     info->last_path = h->last_path;

@@ -103,6 +103,8 @@ cudaError_t launch_update_touched64(bool adagrad, float* w, float* Gacc, double*
 cudaError_t launch_grad_export(double* g, float* out, int64_t M, int sm_count, cudaStream_t st);
 // Clears the bitmap words of the listed starts and resets the list count.
 cudaError_t launch_touched_clear(const Touched& touched, int sm_count, cudaStream_t st);
+// Circular array: g[z] += g[M + z], g[M + z] = 0 for z < L (g64 or g32).
+cudaError_t launch_fold_tail(double* g64, float* g32, int64_t M, int L, cudaStream_t st);
 // direction 0: fp32 -> fp64 (widen); 1: fp64 -> fp32 (narrow), n values.
 cudaError_t launch_convert(int direction, const void* in, void* out, int64_t n, int sm_count,
                            cudaStream_t st);

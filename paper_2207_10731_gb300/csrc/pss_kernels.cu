@@ -127,6 +127,21 @@ k_update_dense(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g
     }
 }
 
+// Circular array: the gradient accumulator has L elements past M that stand
+// for M[0 .. L) (blocks near the end wrap there); fold them into the head and
+// clear them.
+template <typename GT>
+__global__ void __launch_bounds__(kThreads) k_fold_tail(GT* __restrict__ g, int64_t M, int L) {
+    pdl_prologue();
+    for (int z = blockIdx.x * blockDim.x + threadIdx.x; z < L; z += gridDim.x * blockDim.x) {
+        const GT v = g[M + z];
+        if (nonzero(v)) {
+            g[z] += v;
+            g[M + z] = (GT)0;
+        }
+    }
+}
+
 // Conversion check: the integer fp32 <-> fp64 conversions of the accumulation
 // path applied to n values.
 __global__ void __launch_bounds__(kThreads)
@@ -274,6 +289,12 @@ cudaError_t launch_update_touched64(bool adagrad, float* w, float* Ga, double* g
 cudaError_t launch_grad_export(double* g, float* out, int64_t M, int sm_count, cudaStream_t st) {
     const int grid = grid_for(k_grad_export, sm_count, (M + kThreads - 1) / kThreads);
     return launch_k(k_grad_export, dim3(grid), dim3(kThreads), 0, st, g, out, M);
+}
+
+cudaError_t launch_fold_tail(double* g64, float* g32, int64_t M, int L, cudaStream_t st) {
+    const int grid = (L + kThreads - 1) / kThreads;
+    if (g64) return launch_k(k_fold_tail<double>, dim3(grid), dim3(kThreads), 0, st, g64, M, L);
+    return launch_k(k_fold_tail<float>, dim3(grid), dim3(kThreads), 0, st, g32, M, L);
 }
 
 cudaError_t launch_convert(int direction, const void* in, void* out, int64_t n, int sm_count,

@@ -510,6 +510,97 @@ def test_signed_option_forgets_the_batch_and_needs_small_R():
 
 
 # --------------------------------------------------------------------------
+# circular array (NEXT row: R = M/G starts, blocks past M wrap to its start)
+CIRC_CASES = [
+    dict(name="tiny", M=256),                 # 64 starts, 3 of them wrap
+    dict(name="tiny"),
+    dict(name="kaggle"),
+    dict(name="tb", B=4096),
+    dict(name="multihot", B=1024),
+    dict(name="tiny", Z=1, G=1, M=999),       # scalar kernels
+    dict(name="kaggle", Z=3, G=2, B=300),     # Z does not divide d
+]
+
+
+def _circ_pair(w, path, signed=False):
+    from oracle import OraclePSS
+    h, _ = gu.make_pair(w)
+    o = OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, signed=signed, circular=True)
+    o_abs = OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, circular=True)
+    h.set_option(binding.OPT_CIRCULAR, 1)
+    if signed:
+        h.set_option(binding.OPT_SIGNED, 1)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    h.set_weights(gu.cuda(w.w0))      # (re)load: refreshes the mirror of M[0 .. L)
+    return h, o, o_abs
+
+
+@pytest.mark.parametrize("signed", [False, True])
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("case", CIRC_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_circular_forward_and_grad_parity(case, path, signed):
+    w = _wl(case)
+    h, o, o_abs = _circ_pair(w, path, signed)
+    info = h.info()
+    assert info["circular"] == 1 and info["R"] == o.R == w.M // w.G
+    np.testing.assert_array_equal(gu.host(h.compute_locations(*_batch_cuda(w), w.B)),
+                                  o.locations(w.indices, w.offsets, w.B)[0])
+    out = gu.host(h.forward(*_batch_cuda(w), w.B)).ravel()
+    ref, bad = o.forward(w.w0, w.indices, w.offsets, w.B)
+    assert bad == -1
+    gu.check_forward(out, ref, _abs_pool(o_abs, w.w0, w), what="circular forward")
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    gref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
+    A = o_abs.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g, gref, A, what="circular grad")
+    h.close()
+
+
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("opt", ["sgd", "adagrad"])
+def test_circular_steps_dyadic_bit_exact(opt, path):
+    # three steps: each forward reads the wrapped blocks through the mirror the
+    # previous update refreshed; dyadic inputs make every result exact
+    w = wl.make_workload("tiny", M=256, grad="dyadic", w0="dyadic", opt=opt)
+    w.lr = 0.125
+    h, o, _ = _circ_pair(w, path)
+    wcur, Gcur = w.w0.copy(), np.zeros(w.M, np.float32)
+    for k in range(3):
+        wk = wl.make_workload("tiny", M=256, grad="dyadic", w0="dyadic", opt=opt, batch=k)
+        out = gu.host(h.forward(*_batch_cuda(wk), wk.B)).ravel()
+        ref, _ = o.forward(wcur, wk.indices, wk.offsets, wk.B)
+        np.testing.assert_array_equal(out, ref)
+        h.backward_update(gu.cuda(wk.grad_out), w.lr)
+        wcur, Gcur, _ = o.step(wcur, Gcur, wk.indices, wk.offsets, wk.B, wk.grad_out, opt, w.lr,
+                               w.eps)
+        wg, Gg = h.get_state()
+        np.testing.assert_array_equal(gu.host(wg), wcur)
+        if opt == "adagrad":
+            np.testing.assert_array_equal(gu.host(Gg), Gcur)
+    h.close()
+
+
+def test_circular_option_rules():
+    w = wl.make_workload("tiny")
+    h, _ = gu.make_pair(w)
+    R0 = h.info()["R"]
+    h.forward(*_batch_cuda(w), w.B)
+    h.set_option(binding.OPT_CIRCULAR, 1)
+    assert h.info()["R"] == w.M // w.G != R0
+    with pytest.raises(binding.PSSError) as e:
+        h.backward_update(gu.cuda(w.grad_out), w.lr)
+    assert e.value.status == binding.PSS_ERR_STATE
+    h.set_option(binding.OPT_CIRCULAR, 0)
+    assert h.info()["R"] == R0 and h.get_option(binding.OPT_CIRCULAR) == 0
+    h.close()
+    odd = binding.PSS(w.cards, dim=16, M=1002, Z=16, G=4, seed=0, optimizer="sgd")
+    with pytest.raises(binding.PSSError) as e:
+        odd.set_option(binding.OPT_CIRCULAR, 1)
+    assert e.value.status == binding.PSS_ERR_UNSUPPORTED
+    odd.close()
+
+
+# --------------------------------------------------------------------------
 # host buffers through the same C-ABI calls (the end-to-end path)
 def test_host_buffers_match_device_buffers():
     # dyadic inputs: every sum is exact, so both paths must give the same bits
