@@ -209,6 +209,18 @@ def _oracle_rate(w: wl.Workload, budget_s: float, forward_only: bool = False,
     return lookups / tot, rows, reps, idx.shape[0], tot
 
 
+def reduce_over_ranks(dist, device, elapsed_ms: float, work: float):
+    """Replicas: the job's time is the slowest rank's timed region, its work
+    the sum over ranks (one all-reduce each; the process group may be NCCL on
+    GPUs or gloo on the host)."""
+    import torch
+    t = torch.tensor([elapsed_ms, float(work)], dtype=torch.float64, device=device)
+    tmax = t.clone()
+    dist.all_reduce(tmax[:1], op=dist.ReduceOp.MAX)
+    dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
+    return float(tmax[0]), float(t[1])
+
+
 def _shape_overrides(args):
     """Chunk size Z and offset alignment G given on the command line."""
     return {k: v for k, v in (("Z", args.Z), ("G", args.G)) if v is not None}
@@ -374,11 +386,7 @@ def run_gpu(args):
         sampler.stop()
     lookups = sum(nnz_per_step[k % len(nnz_per_step)] for k in range(args.steps))
     if world > 1:
-        t = torch.tensor([elapsed_ms, float(lookups)], dtype=torch.float64, device=dev)
-        tmax = t.clone()
-        dist.all_reduce(tmax[:1], op=dist.ReduceOp.MAX)
-        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
-        elapsed_ms, lookups = float(tmax[0]), float(t[1])
+        elapsed_ms, lookups = reduce_over_ranks(dist, dev, elapsed_ms, lookups)
 
     # end to end through the same C-ABI calls with pinned HOST buffers:
     # every step copies indices, offsets and grad_out in and the pooled output out.
@@ -406,11 +414,7 @@ def run_gpu(args):
     e2e_ms = e0.elapsed_time(e1)
     e2e_lookups = sum(nnz_per_step[k % len(nnz_per_step)] for k in range(e2e_steps))
     if world > 1:
-        t = torch.tensor([e2e_ms, float(e2e_lookups)], dtype=torch.float64, device=dev)
-        tmax = t.clone()
-        dist.all_reduce(tmax[:1], op=dist.ReduceOp.MAX)
-        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
-        e2e_ms, e2e_lookups = float(tmax[0]), float(t[1])
+        e2e_ms, e2e_lookups = reduce_over_ranks(dist, dev, e2e_ms, e2e_lookups)
     h2d = int(np.mean([i.nbytes + o.nbytes + (0 if args.forward_only else g.nbytes)
                        for i, o, g in batches]))
     d2h = int(hout.numel() * 4)
