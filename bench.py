@@ -222,8 +222,11 @@ def reduce_over_ranks(dist, device, elapsed_ms: float, work: float):
 
 
 def _shape_overrides(args):
-    """Chunk size Z and offset alignment G given on the command line."""
-    return {k: v for k, v in (("Z", args.Z), ("G", args.G)) if v is not None}
+    """Chunk size Z, offset alignment G and id distribution given on the command line."""
+    over = {k: v for k, v in (("Z", args.Z), ("G", args.G)) if v is not None}
+    if args.ids == "uniform":
+        over["ids"] = ("uniform",)
+    return over
 
 
 def _config_extra(args, w):
@@ -235,6 +238,8 @@ def _config_extra(args, w):
         extra["mode"] = "forward only (inference): hash + gather + sum-pool, no backward"
     if args.signed:
         extra["signed_hash"] = True
+    if args.ids == "uniform":
+        extra["ids"] = "uniform over each table"
     return extra
 
 
@@ -309,7 +314,9 @@ def run_gpu(args):
     batches = [(w.indices, w.offsets, w.grad_out)]
     for k in range(1, args.rotate):
         batches.append(wl.make_batch(w.cards, w.B, w.d, wl.CONFIGS[args.workload]["bag"],
-                                     wl.CONFIGS[args.workload]["ids"], seed=rank, batch=k,
+                                     _shape_overrides(args).get("ids",
+                                                                wl.CONFIGS[args.workload]["ids"]),
+                                     seed=rank, batch=k,
                                      grad=wl.CONFIGS[args.workload].get("grad", "normal")))
     dbatches = [(torch.from_numpy(i).to(dev), torch.from_numpy(o).to(dev),
                  torch.from_numpy(g).to(dev)) for i, o, g in batches]
@@ -506,6 +513,9 @@ def main(argv=None):
     ap.add_argument("--forward-only", action="store_true",
                     help="time the forward (inference) alone")
     ap.add_argument("--signed", action="store_true", help="signed hashing (PSS_OPT_SIGNED)")
+    ap.add_argument("--ids", choices=["workload", "uniform"], default="workload",
+                    help="id distribution: the workload's own (Zipf for the Criteo shapes) or "
+                         "uniform over each table")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")

@@ -85,7 +85,9 @@ typedef enum {
     /* Backward path: the dense gradient of Algorithm 1 built with vector atomics
      * (PSS_PATH_ATOMIC), or the sorted, deterministic path that reduces equal
      * locations before touching M (PSS_PATH_SORTED, Algorithm 1's sparse branch).
-     * PSS_PATH_AUTO picks by the measured collision rate of the previous batch. */
+     * PSS_PATH_AUTO takes the sorted path when the batch adds at least 2^23
+     * elements (nnz * J * L), the atomic one below (crossover measured on
+     * GB300; M does not move it). */
     PSS_OPT_BACKWARD_PATH = 1,
     /* How the Adagrad step visits M: every element (PSS_UPDATE_DENSE), only the
      * blocks the batch touched (PSS_UPDATE_TOUCHED), or chosen from M and the
@@ -123,7 +125,15 @@ typedef enum {
      * is then always the dense one.  Changing it synchronises the device,
      * changes R (pss_get_info) and forgets the last forward's batch.
      * pss_grad_noalloc does not wrap. */
-    PSS_OPT_CIRCULAR = 7
+    PSS_OPT_CIRCULAR = 7,
+    /* log2 of the number of counters of the sorted path's counting sort, 4 to
+     * 30 (default 22).  With more block starts R than counters, block x is
+     * counted under x mod 2^value: the counters stay small enough to live in
+     * L2 at any M, and entries come out grouped by residue, runs of buckets
+     * that share one alternating within a group (the reduce checks every
+     * entry then).  Results do not depend on it.  Changing it synchronises
+     * the device and forgets the last forward's batch. */
+    PSS_OPT_SORT_KEYS = 8
 } pss_option;
 
 
@@ -152,7 +162,10 @@ typedef struct {
     int64_t optimizer;         /* pss_optimizer */
     int64_t kernel_launches;   /* kernels this handle has launched so far */
     int64_t last_path;         /* PSS_PATH_ATOMIC / PSS_PATH_SORTED of the last backward */
-    double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass, or -1 */
+    double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass, or -1;
+                                  with R > 2^22 the distinct residues of the block index
+                                  mod 2^22 stand in for the distinct blocks (an upper
+                                  bound on the rate) */
     uint64_t A2, B2;           /* sign-hash parameters derived from the seed */
     int64_t signed_hash;       /* PSS_OPT_SIGNED */
     int64_t circular;          /* PSS_OPT_CIRCULAR */

@@ -64,6 +64,7 @@ struct pss_handle {
     int64_t profile = 0;
     int64_t sync_check = 0;
     int64_t accum = PSS_ACCUM_F64;
+    int64_t sort_keys_log2 = 22;                // PSS_OPT_SORT_KEYS
     int64_t last_path = PSS_PATH_ATOMIC;
     double last_collision = -1.0;
 
@@ -334,10 +335,17 @@ bool use_touched(const pss_handle* h, int64_t pairs) {
     return h->dp.M > pairs * (int64_t)h->dp.L;
 }
 
-// Largest bucket count for which the sorted path keeps per-bucket counters
-// (4 bytes each, twice); AUTO takes the sorted path up to kAutoSortedMaxR.
-constexpr int64_t kSortedMaxR = int64_t(1) << 28;
-constexpr int64_t kAutoSortedMaxR = int64_t(1) << 26;
+// The sorted path holds bucket indices in 32 bits, 0xffffffff marking a bad
+// id; above 2^sort_keys_log2 buckets its counters are shared by residue (see
+// SortedBuffers).  AUTO takes the sorted path when the batch adds at least
+// kAutoSortedMinAdds elements (pairs * L): measured on GB300, the atomic path
+// wins below it (its one kernel against the sort's five; Criteo-Kaggle shape
+// at batch 8192: 3.4M adds, 0.049 against 0.108 ms per step), the sorted path
+// above it at every M from 2^18 to 2^33, Zipf or uniform ids (Criteo-Kaggle
+// shape at batch 32768 and Criteo-TB shape at batch 4096: 13.6M adds, 0.138
+// against 0.186 and 0.073 against 0.113 ms).
+constexpr int64_t kSortedMaxR = int64_t(0xffffffffLL);
+constexpr int64_t kAutoSortedMinAdds = int64_t(1) << 23;
 
 bool sorted_supported(const pss_handle* h, int64_t nnz, int64_t B) {
     const int64_t J = h->dp.J;
@@ -348,20 +356,24 @@ bool sorted_supported(const pss_handle* h, int64_t nnz, int64_t B) {
            (int64_t)h->dp.T * B * J < lim;
 }
 
-bool want_sorted(const pss_handle* h) {
+bool want_sorted(const pss_handle* h, int64_t npairs) {
     if (h->path == PSS_PATH_SORTED) return true;
     if (h->path == PSS_PATH_ATOMIC) return false;
-    return (int64_t)h->dp.R <= kAutoSortedMaxR;
+    return npairs * (int64_t)h->dp.L >= kAutoSortedMinAdds;
 }
 
 pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {
     const int64_t R = (int64_t)h->dp.R;
     const int64_t npairs = nnz * h->dp.J;
     if (!h->sb_counters) {
-        const int64_t nblk = sorted_scan_blocks(R);
-        PSS_TRY(cudaMalloc(&h->sb.cnt, sizeof(uint32_t) * (size_t)R));
-        PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)R, st));
-        PSS_TRY(cudaMalloc(&h->sb.start, sizeof(uint32_t) * (size_t)(R + 1)));
+        const int64_t K = int64_t(1) << h->sort_keys_log2;   // residues are taken with a mask
+        const int64_t nkeys = R < K ? R : K;
+        h->sb.nkeys = nkeys;
+        h->sb.kmask = R <= K ? 0xffffffffu : (uint32_t)(K - 1);
+        const int64_t nblk = sorted_scan_blocks(nkeys);
+        PSS_TRY(cudaMalloc(&h->sb.cnt, sizeof(uint32_t) * (size_t)nkeys));
+        PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)nkeys, st));
+        PSS_TRY(cudaMalloc(&h->sb.start, sizeof(uint32_t) * (size_t)(nkeys + 1)));
         PSS_TRY(cudaMalloc(&h->sb.bsum, sizeof(uint32_t) * (size_t)nblk));
         PSS_TRY(cudaMalloc(&h->sb.bnz, sizeof(uint32_t) * (size_t)nblk));
         PSS_TRY(cudaMalloc(&h->sb.stats, 2 * sizeof(unsigned long long)));
@@ -661,7 +673,8 @@ pss_status pss_forward(pss_handle* h, const int64_t* indices, int64_t nnz, const
         PSS_TRY(ensure(h->st_out, nout * sizeof(float), st));
         dout = static_cast<float*>(h->st_out.ptr);
     }
-    const bool emit = nbags > 0 && want_sorted(h) && sorted_supported(h, nnz, B);
+    const bool emit =
+        nbags > 0 && want_sorted(h, nnz * (int64_t)h->dp.J) && sorted_supported(h, nnz, B);
     if (emit && (rc = ensure_sorted(h, nnz, st)) != PSS_OK) return rc;
     if (nbags > 0) {
         LaunchScope ls(h, PSS_K_FORWARD, st);
@@ -710,11 +723,17 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, 
     if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
     poll_stats(h);
     // cnt is zero here: it is zeroed when allocated, and every sort's slot
-    // scatter counts each bucket back down by exactly what its count added
+    // scatter counts each key back down by exactly what its count added.
+    // With counters shared by residue, the touched buckets come from the
+    // pairs themselves rather than from the non-empty counters.
+    const bool mixed = h->sb.kmask != 0xffffffffu;
     {
-        LaunchScope ls(h, PSS_K_SORT, st, 5);
+        LaunchScope ls(h, PSS_K_SORT, st, (touch && mixed) ? 6 : 5);
         PSS_TRY(launch_sorted_count(h->sb, npairs, h->dp.smask, h->sm_count, st));
-        PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, touch ? &h->touched : nullptr, st));
+        PSS_TRY(launch_sorted_scan(h->sb, h->sb.nkeys, (touch && !mixed) ? &h->touched : nullptr,
+                                   st));
+        if (touch && mixed)
+            PSS_TRY(launch_mark_pairs(h->sb, npairs, h->dp.smask, h->touched, h->sm_count, st));
         PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->dp.smask, h->sm_count, st));
     }
     if (!h->stats_pending) {
@@ -745,7 +764,7 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
     if (rc != PSS_OK) return rc;
     const int64_t pairs = h->last_nnz * (int64_t)h->dp.J;
     const bool ada = h->opt == PSS_ADAGRAD;
-    const bool sorted = h->batch_emitted && want_sorted(h);
+    const bool sorted = h->batch_emitted && want_sorted(h, h->last_nnz * (int64_t)h->dp.J);
     h->last_path = sorted ? PSS_PATH_SORTED : PSS_PATH_ATOMIC;
     if (sorted) {
         const int64_t saved = h->accum;
@@ -828,7 +847,7 @@ pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, 
     bool staged = false;
     pss_status rc = stage_grad(h, grad_out, (size_t)nbags * (size_t)h->dp.d, st, &dg, &staged);
     if (rc != PSS_OK) return rc;
-    const bool sorted = h->batch_emitted && want_sorted(h);
+    const bool sorted = h->batch_emitted && want_sorted(h, h->last_nnz * (int64_t)h->dp.J);
     h->last_path = sorted ? PSS_PATH_SORTED : PSS_PATH_ATOMIC;
     if (sorted) {
         const int64_t saved = h->accum;
@@ -915,6 +934,16 @@ pss_status pss_set_option(pss_handle* h, int32_t key, int64_t value) {
             h->dp.smask = m;
             return PSS_OK;
         }
+        case PSS_OPT_SORT_KEYS: {
+            if (value < 4 || value > 30) return PSS_ERR_INVALID_ARG;
+            if (value == h->sort_keys_log2) return PSS_OK;
+            DeviceGuard g(h->device);
+            PSS_TRY(cudaDeviceSynchronize());
+            release_r_buffers(h);
+            h->sort_keys_log2 = value;
+            h->have_batch = false;
+            return PSS_OK;
+        }
     }
     return PSS_ERR_INVALID_ARG;
 }
@@ -929,6 +958,7 @@ pss_status pss_get_option(pss_handle* h, int32_t key, int64_t* value) {
         case PSS_OPT_ACCUM: *value = h->accum; return PSS_OK;
         case PSS_OPT_SIGNED: *value = h->dp.smask ? 1 : 0; return PSS_OK;
         case PSS_OPT_CIRCULAR: *value = h->circ ? 1 : 0; return PSS_OK;
+        case PSS_OPT_SORT_KEYS: *value = h->sort_keys_log2; return PSS_OK;
     }
     return PSS_ERR_INVALID_ARG;
 }

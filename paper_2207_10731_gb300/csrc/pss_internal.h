@@ -47,20 +47,32 @@ struct Touched {
 struct SortedBuffers {
     uint32_t* pair_x;             // nnz*J buckets written by the forward (0xffffffff: bad id)
     uint32_t* q_row;              // nnz output rows b*T + t written by the forward
-    uint32_t* cnt;                // R per-bucket counts, filled by launch_sorted_count
+    uint32_t* cnt;                // nkeys counts per counting key, filled by launch_sorted_count
     uint32_t* start;              // R + 1 bucket starts
     uint32_t* bsum;               // per scan chunk: entries, then their exclusive prefix
     uint32_t* bnz;                // per scan chunk: non-empty buckets
     unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets
-    unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j) in bucket order
+    unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j) in counting-key order
+    // Counting key of bucket x: x & kmask.  With R <= K counters, kmask has
+    // every bit set and the entries come out in bucket order; above it the
+    // K counters cover the residues of x mod K (a power of two), entries are
+    // grouped by residue, and inside a residue class runs of different
+    // buckets may alternate (the reduce then checks every entry of a block).
+    uint32_t kmask;
+    int64_t nkeys;                // number of counters: min(R, K)
 };
 int64_t sorted_scan_blocks(int64_t R);
-// Per-bucket counts of the valid pairs (cnt must be zero on entry).
+// Per-key counts of the valid pairs (cnt must be zero on entry).
 cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
                                 int sm_count, cudaStream_t st);
-// Bucket starts; with `touched`, also the list / bitmap of non-empty buckets.
+// Key starts; with `touched` (only when every bucket has its own counter),
+// also the list / bitmap of non-empty buckets.
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
                                cudaStream_t st);
+// Touched bitmap / list of the buckets of the forward's pairs (the sorted path
+// when counters are shared by residue).
+cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
+                              const Touched& touched, int sm_count, cudaStream_t st);
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
                                   int sm_count, cudaStream_t st);
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,

@@ -6,11 +6,12 @@
 //              for an id outside its table;
 //   q_row[q]   output row b*T + t of the bag that holds id q;
 // Steps (all on the caller's stream):
-//   0. count    cnt[x] = number of valid pairs with bucket x (cnt zeroed by
-//               the caller);
-//   1. scan     start[x] = sum of cnt[y] for y < x (three kernels);
-//               statistics: valid pairs and distinct buckets;
-//   2. scatter  each pair takes a slot in [start[x], start[x+1]) of sorted_e,
+//   0. count    cnt[k] = number of valid pairs with counting key k = x & kmask
+//               (cnt zeroed by the caller; k = x unless R > kSortKeys, see
+//               SortedBuffers);
+//   1. scan     start[k] = sum of cnt[y] for y < k (three kernels);
+//               statistics: valid pairs and distinct keys;
+//   2. scatter  each pair takes a slot in [start[k], start[k+1]) of sorted_e,
 //               which holds (x, r = row*J + j): the bucket and the
 //               upstream-gradient chunk to add (with signed hashing, bit 31 of
 //               pair_x and of r carries the pair's sign, see pss_device.cuh);
@@ -202,9 +203,9 @@ __device__ __forceinline__ void seg_table_init(uint32_t* s_key, uint32_t* s_val)
     }
 }
 
-// cnt[x] += number of valid pairs with bucket x.
+// cnt[k] += number of valid pairs with counting key k = (x without its sign) & kmask.
 __global__ void __launch_bounds__(kSegThreads)
-k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask,
+k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask, uint32_t kmask,
              uint32_t* __restrict__ cnt) {
     pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
@@ -222,7 +223,7 @@ k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask
         __syncthreads();   // the previous segment's table is clear
 #pragma unroll
         for (int i = 0; i < kSegPer; ++i)
-            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i] & ~smask) : 0u;
+            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i] & ~smask & kmask) : 0u;
         __syncthreads();
 #pragma unroll
         for (int k = 0; k < kSegSlots / kSegThreads; ++k) {
@@ -242,13 +243,15 @@ k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask
 }
 
 // Slot of every valid pair: cnt counts back down to zero, each segment taking
-// one contiguous range of every bucket it holds (one atomic per distinct
-// bucket); within the range a pair's place is its rank in the segment table.
+// one contiguous range of its counting key for every bucket it holds (one
+// atomic per distinct bucket); within the range a pair's place is its rank in
+// the segment table, which is keyed by the bucket, so a segment's pairs of one
+// bucket stay together even when several buckets share a key.
 // sorted_e[slot] = x << 32 | row*J + j.
 template <bool SG>
 __global__ void __launch_bounds__(kSegThreads)
 k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
-               int J, int log2J, const uint32_t* __restrict__ start,
+               int J, int log2J, uint32_t kmask, const uint32_t* __restrict__ start,
                uint32_t* __restrict__ cnt, unsigned long long* __restrict__ sorted_e) {
     pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
@@ -277,7 +280,7 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
                     e[i] |= x[i] & 0x80000000u;
                     x[i] &= 0x7fffffffu;
                 }
-                st0[i] = __ldg(start + x[i]);
+                st0[i] = __ldg(start + (x[i] & kmask));
             }
         }
         __syncthreads();   // the previous segment's table is clear
@@ -298,7 +301,7 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
             }
 #pragma unroll
             for (int u = 0; u < kSegFlushU; ++u)
-                old[u] = (key[u] != kEmpty) ? atomicSub(cnt + key[u], c[u]) : 0u;
+                old[u] = (key[u] != kEmpty) ? atomicSub(cnt + (key[u] & kmask), c[u]) : 0u;
 #pragma unroll
             for (int u = 0; u < kSegFlushU; ++u)
                 if (key[u] != kEmpty) s_val[(k0 + u) * kSegThreads + threadIdx.x] = old[u] - c[u];
@@ -320,6 +323,52 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
     }
 }
 
+// Touched bitmap and list of the buckets of all valid pairs.  A CTA takes
+// chunks of kMarkChunk pairs; a bucket already marked costs one load, a new
+// one an atomicOr, and the CTA gathers its new buckets in shared memory and
+// reserves their list places with one atomic per chunk.
+constexpr int kMarkPer = 16;                          // pairs per thread and chunk
+constexpr int kMarkChunk = kThreads * kMarkPer;
+
+__global__ void __launch_bounds__(kThreads)
+k_mark_pairs(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask, Touched tc) {
+    pdl_prologue();
+    __shared__ uint32_t s_new[kMarkChunk];
+    __shared__ uint32_t s_n;
+    __shared__ unsigned long long s_base;
+    const int64_t nchunks = (npairs + kMarkChunk - 1) / kMarkChunk;
+    for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x) {
+        if (threadIdx.x == 0) s_n = 0u;
+        __syncthreads();
+        uint32_t x[kMarkPer], word[kMarkPer];
+#pragma unroll
+        for (int i = 0; i < kMarkPer; ++i) {
+            const int64_t p = c * kMarkChunk + i * kThreads + threadIdx.x;
+            x[i] = (p < npairs) ? __ldg(pair_x + p) : kBad;
+        }
+#pragma unroll
+        for (int i = 0; i < kMarkPer; ++i) {
+            if (x[i] != kBad) x[i] &= ~smask;
+            word[i] = (x[i] != kBad) ? __ldcg(tc.bitmap + (x[i] >> 5)) : ~0u;
+        }
+#pragma unroll
+        for (int i = 0; i < kMarkPer; ++i) {
+            const uint32_t bit = 1u << (x[i] & 31u);
+            if (!(word[i] & bit) && !(atomicOr(tc.bitmap + (x[i] >> 5), bit) & bit))
+                s_new[atomicAdd(&s_n, 1u)] = x[i];
+        }
+        __syncthreads();
+        const uint32_t n = s_n;
+        if (threadIdx.x == 0) s_base = n ? atomicAdd(tc.count, (unsigned long long)n) : 0ull;
+        __syncthreads();
+        for (uint32_t k = threadIdx.x; k < n; k += kThreads) {
+            const unsigned long long slot = s_base + k;
+            if ((int64_t)slot < tc.cap) tc.list[slot] = (int64_t)s_new[k];
+        }
+        __syncthreads();   // s_new and s_n are reused by the next chunk
+    }
+}
+
 // Reduce: one group of gs lanes per task of kPiece sorted entries; lane lg
 // owns columns lg + k*gs of VW elements of the L-element block.  Each run of
 // equal x is summed with compensation (Kahan) and added once into the fp64
@@ -332,7 +381,7 @@ __global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
 k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                const unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
-               uint32_t smask, double* __restrict__ g, int log2gs) {
+               uint32_t smask, bool mixed, double* __restrict__ g, int log2gs) {
     pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
@@ -430,8 +479,11 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                         for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
                 }
             }
-            if (xs[kRU - 1] == cur) {
-                // the whole block continues the current run (keys are sorted):
+            // the whole block continues the current run when its last entry
+            // does (entries in bucket order), or, when runs of buckets that
+            // share a counting key may alternate, when every entry does
+            if (xs[kRU - 1] == cur &&
+                (!mixed || (xs[0] == cur && xs[1] == cur && xs[2] == cur))) {
                 // a tree sum, then one compensated add
 #pragma unroll
                 for (int k = 0; k < KC; ++k)
@@ -476,7 +528,7 @@ __global__ void __launch_bounds__(kThreads)
 k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     const unsigned long long* __restrict__ stats, int64_t npairs,
                     const float* __restrict__ gout, int d, int Z, int J, int log2J, int L,
-                    int64_t G, uint32_t smask, double* __restrict__ g) {
+                    int64_t G, uint32_t smask, bool mixed, double* __restrict__ g) {
     pdl_prologue();
     __shared__ unsigned long long s_ent[kWarps][kPiece];
     const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
@@ -532,7 +584,12 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     v[u][k] = (xs[u] != kBad && z < Lj) ? sign_by(__ldcs(src + z), sb) : 0.f;
                 }
             }
-            if (xs[kWU - 1] == cur) {
+            bool cont = xs[kWU - 1] == cur;
+            if (mixed) {
+#pragma unroll
+                for (int u = 0; u < kWU - 1; ++u) cont = cont && xs[u] == cur;
+            }
+            if (cont) {
 #pragma unroll
                 for (int k = 0; k < KE; ++k) {
                     const float a = (v[0][k] + v[1][k]) + (v[2][k] + v[3][k]);
@@ -583,7 +640,7 @@ __device__ __forceinline__ void cp_async_wait() {
 __global__ void __launch_bounds__(kThreads)
 k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                const unsigned long long* __restrict__ stats, int64_t npairs,
-               const float* __restrict__ gout, int64_t G, uint32_t smask,
+               const float* __restrict__ gout, int64_t G, uint32_t smask, bool mixed,
                double* __restrict__ g) {
     pdl_prologue();
     __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
@@ -651,7 +708,12 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
                 for (int i = 0; i < kAS; ++i) v[i] = sign_by(v[i], ex[2 * i - 1] & smask);
             }
-            if (xlast == cur) {
+            // with alternating runs (buckets sharing a counting key) every
+            // entry of the stage is compared, one per lane
+            const bool cont =
+                xlast == cur &&
+                (!mixed || __all_sync(0xffffffffu, ex[2 * (lane & (kAS - 1))] == cur));
+            if (cont) {
                 const float a = (v[0] + v[1]) + (v[2] + v[3]);
                 const float b = (v[4] + v[5]) + (v[6] + v[7]);
                 kahan_add(sum, comp, a + b);
@@ -686,7 +748,7 @@ cudaError_t warp_reduce_launch(const SortedBuffers& sb, int64_t npairs, const fl
                               (ntasks + kWarps - 1) / kWarps);
     return launch_k(k_warp_range_reduce<KE, ZDIV, JPOW2>, dim3(grid), dim3(kThreads), 0, st,
                     sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask,
-                    g);
+                    sb.kmask != 0xffffffffu, g);
 }
 
 template <int KE>
@@ -710,8 +772,8 @@ cudaError_t reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* 
     const int64_t work_blocks = (ntasks + gpc - 1) / gpc;
     const int grid = grid_for(k_range_reduce<VW, KC, JPOW2, ZDIV>, sm_count, work_blocks, smem);
     return launch_k(k_range_reduce<VW, KC, JPOW2, ZDIV>, dim3(grid), dim3(kThreads), smem, st,
-                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g,
-                    log2gs);
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask,
+                    sb.kmask != 0xffffffffu, g, log2gs);
 }
 
 template <int VW, int KC>
@@ -754,11 +816,11 @@ cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J
     if (smask) {
         const int grid = grid_for(k_sort_scatter<true>, sm_count, nseg);
         return launch_k(k_sort_scatter<true>, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x,
-                        npairs, sb.q_row, J, log2J, sb.start, sb.cnt, sb.sorted_e);
+                        npairs, sb.q_row, J, log2J, sb.kmask, sb.start, sb.cnt, sb.sorted_e);
     }
     const int grid = grid_for(k_sort_scatter<false>, sm_count, nseg);
     return launch_k(k_sort_scatter<false>, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs,
-                    sb.q_row, J, log2J, sb.start, sb.cnt, sb.sorted_e);
+                    sb.q_row, J, log2J, sb.kmask, sb.start, sb.cnt, sb.sorted_e);
 }
 
 cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
@@ -766,7 +828,15 @@ cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_
     const int64_t nseg = (npairs + kSeg - 1) / kSeg;
     const int grid = grid_for(k_sort_count, sm_count, nseg);
     return launch_k(k_sort_count, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs, smask,
-                    sb.cnt);
+                    sb.kmask, sb.cnt);
+}
+
+cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
+                              const Touched& touched, int sm_count, cudaStream_t st) {
+    const int64_t chunks = (npairs + kMarkChunk - 1) / kMarkChunk;
+    const int grid = grid_for(k_mark_pairs, sm_count, chunks);
+    return launch_k(k_mark_pairs, dim3(grid), dim3(kThreads), 0, st, sb.pair_x, npairs, smask,
+                    touched);
 }
 
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
@@ -776,7 +846,7 @@ cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const 
         const int64_t ntasks = (npairs + kAPiece - 1) / kAPiece;   // upper bound
         const int grid = grid_for(k_async_reduce, sm_count, (ntasks + kWarps - 1) / kWarps);
         return launch_k(k_async_reduce, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e, sb.stats,
-                        npairs, gout, p.G, p.smask, g);
+                        npairs, gout, p.G, p.smask, sb.kmask != 0xffffffffu, g);
     }
     // blocks of 32+ elements: one warp per task, one element per lane
     if (p.L >= 32) {

@@ -356,15 +356,22 @@ def _sub_batch(w, rows):
     return np.concatenate(idx_parts).astype(np.int64), off
 
 
-@pytest.mark.parametrize("logM", [18, 20, 22, 24, 26, 28, 30, 32, 33])
-def test_compression_sweep(logM):
+SWEEP = ([(lm, "auto") for lm in (18, 20, 22, 24, 26, 28, 30, 32, 33)] +
+         [(lm, "atomic") for lm in (28, 30, 32, 33)])
+
+
+@pytest.mark.parametrize("logM,path", SWEEP, ids=[f"2^{lm}-{p}" for lm, p in SWEEP])
+def test_compression_sweep(logM, path):
     """Criteo-TB shape with M from 2^18 to 2^33 fp32 (1 MB .. 32 GB).  Up to
     2^26 everything is compared; above, sampled rows and sampled elements
-    (touched and untouched) are compared with the oracle evaluated one by one."""
+    (touched and untouched) are compared with the oracle evaluated one by one.
+    AUTO takes the sorted path here (above 2^22 block starts its counters are
+    shared by residue); the atomic path is forced at the large sizes too."""
     t = gu.torch()
     M = 1 << logM
     w = wl.make_workload("sweep", M=M)
     h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
     idx, off = _batch_cuda(w)
     out = h.forward(idx, off, w.B)
     rng = np.random.default_rng(logM)
@@ -419,9 +426,101 @@ def test_compression_sweep(logM):
         gu.check_adagrad(gu.host(wg[sel]), gu.host(Gg[sel]), w_s, G_s, g32, A_at, w.lr,
                          what=f"sweep 2^{logM} sampled")
         del wg, Gg
+    assert h.info()["last_path"] == (binding.PATH_ATOMIC if path == "atomic" else
+                                     binding.PATH_SORTED)
     assert h.get_error() == (binding.PSS_OK, -1)
     h.close()
     t.cuda.empty_cache()
+
+
+# --------------------------------------------------------------------------
+# sorted path with counters shared by residue (more block starts than
+# counters): a small counter count puts hundreds of buckets on each counter,
+# so runs of different buckets alternate inside every residue group
+RESIDUE_CASES = [
+    dict(name="tb", B=2048),                                  # 32-float chunks, staged reduce
+    dict(name="multihot", B=256),                             # multi-id bags
+    dict(name="multihot", B=301, bag=("uniform", 0, 6)),      # empty bags, ragged tail
+    dict(name="tb", B=300, d=200, Z=32),                      # warp reduce, short last chunk
+    dict(name="kaggle", Z=3, G=2, B=300),                     # lane-group reduce
+    dict(name="tiny", Z=1, G=1),                              # one element per block
+]
+
+
+@pytest.mark.parametrize("keys", [4, 10])
+@pytest.mark.parametrize("signed", [False, True], ids=["unsigned", "signed"])
+@pytest.mark.parametrize("case", RESIDUE_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_sorted_residue_keys_parity(case, signed, keys):
+    from oracle import OraclePSS
+    w = _wl(case)
+    h, o_u = gu.make_pair(w)
+    o = o_u
+    if signed:
+        o = OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, signed=True)
+        h.set_option(binding.OPT_SIGNED, 1)
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    h.set_option(binding.OPT_SORT_KEYS, keys)
+    assert h.get_option(binding.OPT_SORT_KEYS) == keys
+    assert h.info()["R"] > (1 << keys)
+    idx, off = _batch_cuda(w)
+    out = gu.host(h.forward(idx, off, w.B)).ravel()
+    ref, _ = o.forward(w.w0, w.indices, w.offsets, w.B)
+    gu.check_forward(out, ref, _abs_pool(o_u, w.w0, w), what="residue forward")
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    A = o_u.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, w.grad_out), A, what="residue grad")
+    assert h.info()["last_path"] == binding.PATH_SORTED
+    # a step with each update pass: the touched one lists the buckets from the pairs
+    for mode in (binding.UPDATE_TOUCHED, binding.UPDATE_DENSE):
+        h.set_state(gu.cuda(w.w0), gu.cuda(np.zeros(w.M, np.float32)) if w.opt == "adagrad" else None)
+        h.set_option(binding.OPT_UPDATE_MODE, mode)
+        wg, Gg, w2, G2, g32, _ = _run_step(w, h, o, w.w0, np.zeros(w.M, np.float32),
+                                           (w.indices, w.offsets, w.grad_out))
+        if w.opt == "sgd":
+            gu.check_sgd(wg, w2, A, w.lr, what=f"residue sgd, update mode {mode}")
+        else:
+            gu.check_adagrad(wg, Gg, w2, G2, g32, A, w.lr, what=f"residue adagrad, update mode {mode}")
+    assert h.get_error() == (binding.PSS_OK, -1)
+    h.close()
+
+
+@pytest.mark.parametrize("opt", ["sgd", "adagrad"])
+def test_sorted_residue_keys_dyadic_bit_exact(opt):
+    # dyadic inputs: every sum is exact, so alternating runs must still give
+    # the oracle's bits
+    w = wl.make_workload("kaggle", B=1024, grad="dyadic", w0="dyadic")
+    w.lr = 0.125
+    h, o = gu.make_pair(w, opt=opt)
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    h.set_option(binding.OPT_SORT_KEYS, 6)
+    h.forward(*_batch_cuda(w), w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    wg, Gg = h.get_state()
+    w2, G2, _ = o.step(w.w0, np.zeros(w.M, np.float32), w.indices, w.offsets, w.B, w.grad_out,
+                       opt, w.lr, w.eps)
+    np.testing.assert_array_equal(gu.host(wg), w2)
+    if opt == "adagrad":
+        np.testing.assert_array_equal(gu.host(Gg), G2)
+    h.close()
+
+
+def test_sort_keys_option_rules():
+    w = wl.make_workload("tiny")
+    h, _ = gu.make_pair(w)
+    assert h.get_option(binding.OPT_SORT_KEYS) == 22
+    for bad in (3, 31, -1):
+        with pytest.raises(binding.PSSError) as e:
+            h.set_option(binding.OPT_SORT_KEYS, bad)
+        assert e.value.status == binding.PSS_ERR_INVALID_ARG
+    h.forward(*_batch_cuda(w), w.B)
+    h.set_option(binding.OPT_SORT_KEYS, 22)          # unchanged: the batch stays
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    h.forward(*_batch_cuda(w), w.B)
+    h.set_option(binding.OPT_SORT_KEYS, 8)           # changed: the batch is forgotten
+    with pytest.raises(binding.PSSError) as e:
+        h.backward_update(gu.cuda(w.grad_out), w.lr)
+    assert e.value.status == binding.PSS_ERR_STATE
+    h.close()
 
 
 # --------------------------------------------------------------------------
