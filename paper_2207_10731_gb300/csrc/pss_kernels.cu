@@ -168,10 +168,26 @@ k_grad_export(double* __restrict__ g, float* __restrict__ out, int64_t M) {
     }
 }
 
-// Touched-block pass: one warp per distinct block start x (from the scatter's
-// list).  Element e = x*G + z belongs to the LAST marked start at or below it
-// (no marked bucket in (x, x + z/G]), so every element is updated exactly
-// once and without atomics even though blocks overlap when G < L.
+// Touched-block pass: one warp per kTU distinct block starts x at a time
+// (from the list), their loads in flight together.  Element e = x*G + z
+// belongs to the LAST marked start at or below it (no marked bucket in
+// (x, x + z/G]), so every element is updated exactly once and without atomics
+// even though blocks overlap when G < L.
+constexpr int kTU = 4;
+
+__device__ __forceinline__ bool owns(const uint32_t* __restrict__ bitmap, uint64_t x, int nb) {
+    for (int m0 = 1; m0 <= nb; m0 += 32) {
+        const uint64_t y = x + (uint64_t)m0;
+        const uint64_t w0 = bitmap[y >> 5];
+        const uint64_t w1 = bitmap[(y >> 5) + 1];
+        const uint64_t win = ((w1 << 32) | w0) >> (y & 31);
+        const int cnt = (nb - m0 + 1) < 32 ? (nb - m0 + 1) : 32;
+        const uint64_t mask = (cnt >= 32) ? 0xffffffffull : ((1ull << cnt) - 1);
+        if (win & mask) return false;
+    }
+    return true;
+}
+
 template <bool ADA, typename GT>
 __global__ void __launch_bounds__(kThreads)
 k_update_touched(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__ g,
@@ -180,32 +196,50 @@ k_update_touched(float* __restrict__ w, float* __restrict__ Ga, GT* __restrict__
     const int lane = threadIdx.x & 31;
     unsigned long long n = *tc.count;
     if ((int64_t)n > tc.cap) n = (unsigned long long)tc.cap;
-    const int64_t stride = (int64_t)gridDim.x * kWarps;
-    for (int64_t it = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5); it < (int64_t)n;
+    const int64_t stride = (int64_t)gridDim.x * kWarps * kTU;
+    for (int64_t it = ((int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5)) * kTU; it < (int64_t)n;
          it += stride) {
-        const uint64_t x = (uint64_t)tc.list[it];
+        uint64_t x[kTU];
+        bool valid[kTU];
+#pragma unroll
+        for (int u = 0; u < kTU; ++u) {
+            valid[u] = it + u < (int64_t)n;
+            x[u] = valid[u] ? (uint64_t)tc.list[it + u] : 0ull;
+        }
         for (int z = lane; z < L; z += 32) {
             const int nb = (int)(z / G);   // following starts that could also cover e
-            bool owner = true;
-            for (int m0 = 1; m0 <= nb && owner; m0 += 32) {
-                const uint64_t y = x + (uint64_t)m0;
-                const uint64_t w0 = tc.bitmap[y >> 5];
-                const uint64_t w1 = tc.bitmap[(y >> 5) + 1];
-                const uint64_t win = ((w1 << 32) | w0) >> (y & 31);
-                const int cnt = (nb - m0 + 1) < 32 ? (nb - m0 + 1) : 32;
-                const uint64_t mask = (cnt >= 32) ? 0xffffffffull : ((1ull << cnt) - 1);
-                if (win & mask) owner = false;
+            bool own[kTU];
+            GT raw[kTU];
+#pragma unroll
+            for (int u = 0; u < kTU; ++u) own[u] = valid[u] && owns(tc.bitmap, x[u], nb);
+#pragma unroll
+            for (int u = 0; u < kTU; ++u) raw[u] = own[u] ? g[(int64_t)x[u] * G + z] : (GT)0;
+            float wv[kTU], gav[kTU];
+#pragma unroll
+            for (int u = 0; u < kTU; ++u) {
+                wv[u] = gav[u] = 0.f;
+                if (nonzero(raw[u])) {
+                    const int64_t e = (int64_t)x[u] * G + z;
+                    wv[u] = w[e];
+                    if (ADA) gav[u] = Ga[e];
+                }
             }
-            if (!owner) continue;
-            const int64_t e = (int64_t)x * G + z;
-            const GT raw = g[e];
-            if (!nonzero(raw)) continue;
-            const float gv = to_f32(raw);
-            if (gv != 0.f) {
-                if (ADA) adagrad_elem(w[e], Ga[e], gv, lr, eps);
-                else sgd_elem(w[e], gv, lr);
+#pragma unroll
+            for (int u = 0; u < kTU; ++u) {
+                if (!nonzero(raw[u])) continue;
+                const int64_t e = (int64_t)x[u] * G + z;
+                const float gv = to_f32(raw[u]);
+                if (gv != 0.f) {
+                    if (ADA) {
+                        adagrad_elem(wv[u], gav[u], gv, lr, eps);
+                        Ga[e] = gav[u];
+                    } else {
+                        sgd_elem(wv[u], gv, lr);
+                    }
+                    w[e] = wv[u];
+                }
+                g[e] = (GT)0;
             }
-            g[e] = (GT)0;
         }
     }
 }
@@ -230,7 +264,8 @@ cudaError_t update_dense_inst(float* w, float* Ga, GT* g, int64_t M, float lr, f
 template <bool ADA, typename GT>
 cudaError_t update_touched_inst(float* w, float* Ga, GT* g, const Touched& tc, int64_t G,
                                 int32_t L, float lr, float eps, int sm_count, cudaStream_t st) {
-    const int grid = grid_for(k_update_touched<ADA, GT>, sm_count, (tc.cap + kWarps - 1) / kWarps);
+    const int grid = grid_for(k_update_touched<ADA, GT>, sm_count,
+                              (tc.cap + kWarps * kTU - 1) / (kWarps * kTU));
     return launch_k(k_update_touched<ADA, GT>, dim3(grid), dim3(kThreads), 0, st, w, Ga, g, tc, G,
                     L, lr, eps);
 }
