@@ -482,7 +482,14 @@ cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* id
                      const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
                      uint32_t* pair_x, uint32_t* q_row, int sm_count,
                      cudaStream_t st) {
-    const int wb = (32 >> lay.log2gs) * kBagsPerGroup;      // bags per warp tile
+    // bags per warp tile: kU per lane group (kU loads in flight in the one-id
+    // path) and at least 16.  Measured on GB300: 16-bag tiles beat 32 and 64
+    // at the Criteo-TB shape (0.165 against 0.171 and 0.174 ms per forward)
+    // and on multi-id bags (0.385 against 0.419 ms), where the whole warp
+    // takes one bag at a time; the 16-float rows of the Criteo-Kaggle shape
+    // need the kU per group (batch 32768: 0.026 against 0.036 ms).
+    const int groups = 32 >> lay.log2gs;
+    const int wb = groups * kU > 16 ? groups * kU : 16;
     const int tpt = (int)((B + wb - 1) / wb);
     const size_t smem = (size_t)kWarps * ((size_t)(wb + 1) * sizeof(int64_t) +
                                           (size_t)kWarpPairs * sizeof(XT));
