@@ -149,7 +149,9 @@ typedef enum {
     PSS_K_FORWARD = 1,     /* fused hash + gather + sum-pool */
     PSS_K_SCATTER = 2,     /* backward: hash + vector-atomic scatter (+ fused SGD) */
     PSS_K_UPDATE = 3,      /* optimizer pass over M (dense or touched blocks) */
-    PSS_K_SORT = 4,        /* sorted path: bucket count, scan and slot scatter */
+    PSS_K_SORT = 4,        /* sorted path: bucket count, scan, slot scatter (and, with
+                              counters shared by residue and the touched update, the
+                              marking of the touched blocks) */
     PSS_K_REDUCE = 5,      /* sorted path: run sums into the fp64 accumulator */
     PSS_K_MISC = 6,        /* memsets and small helper kernels */
     PSS_K_COUNT = 7

@@ -655,6 +655,23 @@ def test_circular_forward_and_grad_parity(case, path, signed):
     h.close()
 
 
+@pytest.mark.parametrize("signed", [False, True], ids=["unsigned", "signed"])
+@pytest.mark.parametrize("case", [dict(name="tb", B=2048), dict(name="kaggle", Z=3, G=2, B=300)],
+                         ids=["tb", "kaggle-Z3-G2"])
+def test_circular_with_residue_keys(case, signed):
+    # circular array and counters shared by residue (64 counters): the wrapped
+    # blocks' contributions fold into the head after alternating runs
+    w = _wl(case)
+    h, o, o_abs = _circ_pair(w, "sorted", signed)
+    h.set_option(binding.OPT_SORT_KEYS, 6)
+    h.forward(*_batch_cuda(w), w.B)
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    A = o_abs.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, w.grad_out), A, what="circular residue grad")
+    assert h.info()["last_path"] == binding.PATH_SORTED
+    h.close()
+
+
 @pytest.mark.parametrize("path", ["atomic", "sorted"])
 @pytest.mark.parametrize("opt", ["sgd", "adagrad"])
 def test_circular_steps_dyadic_bit_exact(opt, path):
