@@ -623,9 +623,11 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
 // every run's sum once into the fp64 accumulator.
 constexpr int kAS = 8;          // chunks per stage
 constexpr int kAD = 4;          // ring slots (kAD - 1 stages in flight)
-// sorted entries per task (measured: 256 against 128 gave the multi-hot
-// reduce 0.254 against 0.268 ms and the Criteo-TB one 0.209 against 0.209)
-constexpr int kAPiece = 256;
+// sorted entries per task.  Measured: 256 gave the multi-hot reduce 0.254
+// against 0.268 ms and left the Criteo-TB one unchanged, but its 48 KB of
+// shared memory allow one CTA less per SM and a batch of 16384 leaves ~1.4
+// tasks per warp: that reduce took 77 against 57 us.
+constexpr int kAPiece = 128;
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
     const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
