@@ -89,6 +89,14 @@ struct pss_handle {
     cudaStream_t s_h2d = nullptr;
     cudaEvent_t ev_grad_ready = nullptr, ev_grad_free = nullptr, ev_alloc = nullptr;
     bool grad_free_pending = false;
+    // host-to-device copies of one direction run one after another on the
+    // copy engine, so the gradient's upload also waits for the last forward's
+    // staged ids and offsets (ev_inputs): otherwise those small copies queue
+    // behind it and the forward and the output's download start only once
+    // the whole gradient is in (measured: 9.1 ms per Criteo-TB step instead
+    // of the 5.1 ms the two copy directions take together)
+    cudaEvent_t ev_inputs = nullptr;
+    bool inputs_pending = false;
     // circular array: R = M/G starts, blocks past M wrap to its start.  w and
     // the gradient accumulators have L extra elements past M: w's mirror
     // M[0 .. L) (refreshed after every write of w), the accumulators' collect
@@ -156,7 +164,7 @@ pss_status device_view(const T* p, size_t count, Staging& s, cudaStream_t st, co
 pss_status ensure_copy_stream(pss_handle* h) {
     if (h->s_h2d) return PSS_OK;
     PSS_TRY(cudaStreamCreateWithFlags(&h->s_h2d, cudaStreamNonBlocking));
-    for (cudaEvent_t* e : {&h->ev_grad_ready, &h->ev_grad_free, &h->ev_alloc})
+    for (cudaEvent_t* e : {&h->ev_grad_ready, &h->ev_grad_free, &h->ev_alloc, &h->ev_inputs})
         PSS_TRY(cudaEventCreateWithFlags(e, cudaEventDisableTiming));
     return PSS_OK;
 }
@@ -181,6 +189,10 @@ pss_status stage_grad(pss_handle* h, const float* p, size_t count, cudaStream_t 
         PSS_TRY(cudaStreamWaitEvent(h->s_h2d, h->ev_alloc, 0));
     }
     if (h->grad_free_pending) PSS_TRY(cudaStreamWaitEvent(h->s_h2d, h->ev_grad_free, 0));
+    if (h->inputs_pending) {
+        PSS_TRY(cudaStreamWaitEvent(h->s_h2d, h->ev_inputs, 0));
+        h->inputs_pending = false;
+    }
     PSS_TRY(cudaMemcpyAsync(h->st_grad.ptr, p, bytes, cudaMemcpyHostToDevice, h->s_h2d));
     PSS_TRY(cudaEventRecord(h->ev_grad_ready, h->s_h2d));
     *out = static_cast<const float*>(h->st_grad.ptr);
@@ -568,7 +580,7 @@ pss_status pss_destroy(pss_handle* h) {
         if (b) cudaFree(b);
     if (h->stats_host) cudaFreeHost(h->stats_host);
     if (h->stats_ev) cudaEventDestroy(h->stats_ev);
-    for (cudaEvent_t e : {h->ev_grad_ready, h->ev_grad_free, h->ev_alloc})
+    for (cudaEvent_t e : {h->ev_grad_ready, h->ev_grad_free, h->ev_alloc, h->ev_inputs})
         if (e) cudaEventDestroy(e);
     if (h->s_h2d) cudaStreamDestroy(h->s_h2d);
     for (Staging* s : {&h->st_idx, &h->st_off, &h->st_out, &h->st_grad, &h->st_locs})
@@ -666,6 +678,12 @@ pss_status pss_forward(pss_handle* h, const int64_t* indices, int64_t nnz, const
     const int64_t *di = nullptr, *doff = nullptr;
     if ((rc = device_view(indices, (size_t)nnz, h->st_idx, st, &di)) != PSS_OK) return rc;
     if ((rc = device_view(offsets, (size_t)(nbags + 1), h->st_off, st, &doff)) != PSS_OK) return rc;
+    if (di != indices || doff != offsets) {
+        // host batch staged on st: a host gradient's upload waits for it
+        if ((rc = ensure_copy_stream(h)) != PSS_OK) return rc;
+        PSS_TRY(cudaEventRecord(h->ev_inputs, st));
+        h->inputs_pending = true;
+    }
     const size_t nout = (size_t)nbags * (size_t)h->dp.d;
     float* dout = out;
     const bool host_out = nout > 0 && !is_device_ptr(out);
