@@ -20,6 +20,7 @@ import datetime as _dt
 import hashlib
 import json
 import os
+import re
 import subprocess
 import sys
 import threading
@@ -62,15 +63,24 @@ def _peaks():
 _HOST_ONLY = {"pss_api.cu"}
 
 
+def _code_only(src: str) -> str:
+    """Source text without comments and blank lines (the sources keep no comment
+    markers inside string literals)."""
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    lines = (ln.split("//", 1)[0].rstrip() for ln in src.splitlines())
+    return "\n".join(ln for ln in lines if ln)
+
+
 def _kernel_sha():
-    """Hash of the library's device-code sources: the kernels, their launchers
-    and the headers they share (traffic figures go stale with it)."""
+    """Hash of the code of the library's device-code sources: the kernels,
+    their launchers and the headers they share, comments left out (traffic
+    figures go stale with it)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2207_10731_gb300", "csrc")
     for f in sorted(os.listdir(csrc)):
         if f.endswith((".cu", ".cuh", ".h")) and f not in _HOST_ONLY:
-            with open(os.path.join(csrc, f), "rb") as fh:
-                h.update(f.encode() + b"\0" + fh.read())
+            with open(os.path.join(csrc, f), encoding="utf-8") as fh:
+                h.update(f.encode() + b"\0" + _code_only(fh.read()).encode())
     return h.hexdigest()[:16]
 
 

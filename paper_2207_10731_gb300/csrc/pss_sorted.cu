@@ -7,8 +7,8 @@
 //   q_row[q]   output row b*T + t of the bag that holds id q;
 // Steps (all on the caller's stream):
 //   0. count    cnt[k] = number of valid pairs with counting key k = x & kmask
-//               (cnt zeroed by the caller; k = x unless R > kSortKeys, see
-//               SortedBuffers);
+//               (cnt zeroed by the caller; k = x unless R exceeds the number
+//               of counters, see SortedBuffers);
 //   1. scan     start[k] = sum of cnt[y] for y < k (three kernels);
 //               statistics: valid pairs and distinct keys;
 //   2. scatter  each pair takes a slot in [start[k], start[k+1]) of sorted_e,
@@ -21,7 +21,13 @@
 //               compensated (Kahan) fp32 sums, and adds every run's sum once
 //               into the fp64 gradient accumulator g[G*x + z] -- one reduction
 //               per run and element instead of one per contribution, and no
-//               queue of reductions on a hot address.
+//               queue of reductions on a hot address.  With `mixed` (counters
+//               shared by residue) runs of different buckets may alternate,
+//               and a block of entries is summed as one run only when every
+//               entry of it belongs to the current run.
+// With counters shared by residue and the touched update, k_mark_pairs lists
+// the touched blocks from pair_x (the scan cannot: a non-empty counter no
+// longer names one bucket).
 // The optimizer pass over g follows (pss_kernels.cu).
 #include <climits>
 

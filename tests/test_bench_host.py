@@ -65,3 +65,9 @@ def test_binding_option_values_match_the_header():
     assert opts, "no options found in the header"
     for name, value in opts.items():
         assert getattr(binding, "OPT_" + name) == value, name
+
+
+def test_traffic_hash_ignores_comments_and_the_host_only_file():
+    assert bench._code_only("a = 1;  // note\n/* block\n comment */b = 2;\n\n") == "a = 1;\nb = 2;"
+    assert "pss_api.cu" in bench._HOST_ONLY
+    assert len(bench._kernel_sha()) == 16
