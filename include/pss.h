@@ -83,11 +83,13 @@ typedef enum { PSS_SGD = 0, PSS_ADAGRAD = 1 } pss_optimizer;
 /* Option keys for pss_set_option / pss_get_option. */
 typedef enum {
     /* Backward path: the dense gradient of Algorithm 1 built with vector atomics
-     * (PSS_PATH_ATOMIC), or the sorted, deterministic path that reduces equal
-     * locations before touching M (PSS_PATH_SORTED, Algorithm 1's sparse branch).
-     * PSS_PATH_AUTO takes the sorted path when the batch adds at least 2^23
-     * elements (nnz * J * L), the atomic one below (crossover measured on
-     * GB300; M does not move it). */
+     * (PSS_PATH_ATOMIC), or the sorted path that reduces equal locations before
+     * touching M (PSS_PATH_SORTED, Algorithm 1's sparse branch).  In both, the
+     * order of a location's contributions depends on the GPU's scheduling, so
+     * low-order bits may differ between runs (within the accumulation bound;
+     * dyadic inputs give identical bits).  PSS_PATH_AUTO takes the sorted path
+     * when the batch adds at least 2^23 elements (nnz * J * L), the atomic one
+     * below (crossover measured on GB300; M does not move it). */
     PSS_OPT_BACKWARD_PATH = 1,
     /* How the Adagrad step visits M: every element (PSS_UPDATE_DENSE), only the
      * blocks the batch touched (PSS_UPDATE_TOUCHED), or chosen from M and the
@@ -165,9 +167,10 @@ typedef struct {
     int64_t kernel_launches;   /* kernels this handle has launched so far */
     int64_t last_path;         /* PSS_PATH_ATOMIC / PSS_PATH_SORTED of the last backward */
     double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass, or -1;
-                                  with R > 2^22 the distinct residues of the block index
-                                  mod 2^22 stand in for the distinct blocks (an upper
-                                  bound on the rate) */
+                                  with more block starts than sort counters (2^22 unless
+                                  PSS_OPT_SORT_KEYS says otherwise) the distinct residues of
+                                  the block index stand in for the distinct blocks (an
+                                  upper bound on the rate) */
     uint64_t A2, B2;           /* sign-hash parameters derived from the seed */
     int64_t signed_hash;       /* PSS_OPT_SIGNED */
     int64_t circular;          /* PSS_OPT_CIRCULAR */
