@@ -348,8 +348,9 @@ bool use_touched(const pss_handle* h, int64_t pairs) {
 }
 
 // The sorted path holds bucket indices in 32 bits, 0xffffffff marking a bad
-// id; above 2^sort_keys_log2 buckets its counters are shared by residue (see
-// SortedBuffers).  AUTO takes the sorted path when the batch adds at least
+// id: it needs R < kSortedMaxR, the bound below which the forward emits 32-bit
+// buckets at all.  Above 2^sort_keys_log2 buckets its counters are shared by
+// residue (see SortedBuffers).  AUTO takes the sorted path when the batch adds at least
 // kAutoSortedMinAdds elements (pairs * L): measured on GB300, the atomic path
 // wins below it (its one kernel against the sort's five; Criteo-Kaggle shape
 // at batch 8192: 3.4M adds, 0.049 against 0.108 ms per step), the sorted path
@@ -364,7 +365,7 @@ bool sorted_supported(const pss_handle* h, int64_t nnz, int64_t B) {
     // entries hold row*J + j in 32 bits (31 with signed hashing: the sign
     // travels in bit 31)
     const int64_t lim = h->dp.smask ? (int64_t)0x7fffffffLL : (int64_t)0xffffffffLL;
-    return (int64_t)h->dp.R <= kSortedMaxR && nnz * J < (int64_t)0xffffffffLL &&
+    return (int64_t)h->dp.R < kSortedMaxR && nnz * J < (int64_t)0xffffffffLL &&
            (int64_t)h->dp.T * B * J < lim;
 }
 
