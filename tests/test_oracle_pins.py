@@ -545,3 +545,30 @@ def test_grad_at_matches_dense_grad():
     elems = np.unique(np.concatenate([rng.integers(0, w.M, 500), np.flatnonzero(g)[:2000]]))
     ga = o.grad_at(w.indices, w.offsets, w.B, w.grad_out, elems)
     np.testing.assert_allclose(ga, g[elems], rtol=1e-12, atol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# property-based sweep of the brute-force pin: random tiny shapes, including
+# Z > d, Z not dividing d, G > 1 with ragged ranges, empty bags and tables of
+# three ids (hypothesis is optional: the GPU hosts do not ship it)
+def test_forward_and_grad_equal_bruteforce_matrix_random_shapes():
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @hyp.settings(max_examples=60, deadline=None, derandomize=True)
+    @hyp.given(T=st.integers(1, 3), B=st.integers(1, 5), d=st.integers(1, 40),
+               Z=st.integers(1, 48), G=st.integers(1, 8), extra=st.integers(0, 300),
+               max_bag=st.integers(0, 4), seed=st.integers(0, 2**32 - 1))
+    def check(T, B, d, Z, G, extra, max_bag, seed):
+        L = min(Z, d)
+        M = L + extra
+        cards, idx, off, w, go = _tiny_case(seed, T=T, B=B, d=d, M=M, Z=Z, G=G, max_bag=max_bag)
+        o = OraclePSS(cards, d=d, M=M, Z=Z, G=G, seed=seed)
+        P = _bruteforce_P(cards, idx, off, B, d, M, Z, G, seed)
+        out, bad = o.forward(w, idx, off, B)
+        assert bad == -1
+        np.testing.assert_array_equal(out, (P @ w.astype(np.float64)).astype(np.float32))
+        g = o.grad(idx, off, B, go)
+        np.testing.assert_array_equal(g, P.T @ go.astype(np.float64))
+
+    check()
