@@ -572,3 +572,49 @@ def test_forward_and_grad_equal_bruteforce_matrix_random_shapes():
         np.testing.assert_array_equal(g, P.T @ go.astype(np.float64))
 
     check()
+
+
+def _bruteforce_P_variant(cards, idx, offsets, B, d, M, Z, G, seed, signed, circular):
+    """The +-1 (signed) and wrapping (circular) mapping matrices, from big integers."""
+    T = len(cards)
+    A, B0 = bh.params(seed)
+    A2, B2 = bh.sign_params(seed)
+    L, J = min(Z, d), -(-d // Z)
+    R = M // G if circular else (M - L) // G + 1
+    rows, cols, vals = [], [], []
+    for t in range(T):
+        for b in range(B):
+            s = t * B + b
+            for q in range(offsets[s], offsets[s + 1]):
+                i = int(idx[q])
+                for k in range(d):
+                    j, z = divmod(k, Z)
+                    loc = bh.location(A, B0, R, G, T, J, i, t, j)
+                    rows.append((b * T + t) * d + k)
+                    cols.append((loc + z) % M if circular else loc + z)
+                    vals.append(bh.sign(A2, B2, T, J, i, t, j) if signed else 1)
+    return sp.coo_matrix((vals, (rows, cols)), shape=(B * T * d, M)).tocsr()
+
+
+def test_signed_and_circular_variants_equal_bruteforce_random_shapes():
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @hyp.settings(max_examples=60, deadline=None, derandomize=True)
+    @hyp.given(T=st.integers(1, 3), B=st.integers(1, 5), d=st.integers(1, 40),
+               Z=st.integers(1, 48), G=st.integers(1, 8), blocks=st.integers(0, 40),
+               max_bag=st.integers(0, 4), seed=st.integers(0, 2**32 - 1),
+               signed=st.booleans(), circular=st.booleans())
+    def check(T, B, d, Z, G, blocks, max_bag, seed, signed, circular):
+        L = min(Z, d)
+        # circular: G divides M; both readings: M >= L
+        M = G * (-(-L // G) + blocks) if circular else L + blocks * G
+        cards, idx, off, w, go = _tiny_case(seed, T=T, B=B, d=d, M=M, Z=Z, G=G, max_bag=max_bag)
+        o = OraclePSS(cards, d=d, M=M, Z=Z, G=G, seed=seed, signed=signed, circular=circular)
+        P = _bruteforce_P_variant(cards, idx, off, B, d, M, Z, G, seed, signed, circular)
+        out, bad = o.forward(w, idx, off, B)
+        assert bad == -1
+        np.testing.assert_array_equal(out, (P @ w.astype(np.float64)).astype(np.float32))
+        np.testing.assert_array_equal(o.grad(idx, off, B, go), P.T @ go.astype(np.float64))
+
+    check()
