@@ -618,3 +618,29 @@ def test_signed_and_circular_variants_equal_bruteforce_random_shapes():
         np.testing.assert_array_equal(o.grad(idx, off, B, go), P.T @ go.astype(np.float64))
 
     check()
+
+
+@pytest.mark.parametrize("signed", [False, True])
+def test_scatter_and_signs_entry_points_equal_bruteforce(signed):
+    # the lower-level entry points: signs() per (id, chunk) from big integers,
+    # and scatter() of explicit locations (and signs) equal to P^T g
+    T, B, d, M, Z, G = 3, 5, 20, 400, 8, 2
+    for seed in range(3):
+        cards, idx, off, w, go = _tiny_case(seed, T=T, B=B, d=d, M=M, Z=Z, G=G, max_bag=4)
+        o = OraclePSS(cards, d=d, M=M, Z=Z, G=G, seed=seed, signed=signed)
+        A, B0 = bh.params(seed)
+        A2, B2 = bh.sign_params(seed)
+        J, L = -(-d // Z), min(Z, d)
+        R = (M - L) // G + 1
+        locs = np.zeros(idx.shape[0] * J, dtype=np.int64)
+        sg = np.zeros(idx.shape[0] * J, dtype=np.int64)
+        for t in range(T):
+            for q in range(off[t * B], off[(t + 1) * B]):
+                for j in range(J):
+                    locs[q * J + j] = bh.location(A, B0, R, G, T, J, int(idx[q]), t, j)
+                    sg[q * J + j] = bh.sign(A2, B2, T, J, int(idx[q]), t, j)
+        if signed:
+            np.testing.assert_array_equal(o.signs(idx, off, B).astype(np.int64), sg)
+        P = _bruteforce_P_variant(cards, idx, off, B, d, M, Z, G, seed, signed, False)
+        g = o.scatter(locs, off, B, idx.shape[0], go, signs=sg.astype(np.int8) if signed else None)
+        np.testing.assert_array_equal(g, P.T @ go.astype(np.float64))
