@@ -623,7 +623,8 @@ def test_signed_and_circular_variants_equal_bruteforce_random_shapes():
 @pytest.mark.parametrize("signed", [False, True])
 def test_scatter_and_signs_entry_points_equal_bruteforce(signed):
     # the lower-level entry points: signs() per (id, chunk) from big integers,
-    # and scatter() of explicit locations (and signs) equal to P^T g
+    # scatter() of explicit locations (and signs) equal to P^T g, and pool()
+    # of the same equal to P w
     T, B, d, M, Z, G = 3, 5, 20, 400, 8, 2
     for seed in range(3):
         cards, idx, off, w, go = _tiny_case(seed, T=T, B=B, d=d, M=M, Z=Z, G=G, max_bag=4)
@@ -642,5 +643,8 @@ def test_scatter_and_signs_entry_points_equal_bruteforce(signed):
         if signed:
             np.testing.assert_array_equal(o.signs(idx, off, B).astype(np.int64), sg)
         P = _bruteforce_P_variant(cards, idx, off, B, d, M, Z, G, seed, signed, False)
-        g = o.scatter(locs, off, B, idx.shape[0], go, signs=sg.astype(np.int8) if signed else None)
+        s8 = sg.astype(np.int8) if signed else None
+        g = o.scatter(locs, off, B, idx.shape[0], go, signs=s8)
         np.testing.assert_array_equal(g, P.T @ go.astype(np.float64))
+        out = o.pool(w, locs, off, B, idx.shape[0], signs=s8)
+        np.testing.assert_array_equal(out, (P @ w.astype(np.float64)).astype(np.float32))
