@@ -306,7 +306,10 @@ const char* pss_status_string(pss_status s);
  * capture.  Every call shares the one scratch array: calls whose work overlaps
  * on the GPU (other streams, other threads) race and give wrong results, so
  * order them on one stream or synchronise between them.  Asynchronous on
- * `stream`.  Errors: PSS_ERR_INVALID_ARG, PSS_ERR_CAPACITY, PSS_ERR_CUDA.
+ * `stream`: the call queues memsets of the scratch and a few kernels, and the
+ * table sizes travel as kernel arguments, so nothing is copied from host
+ * memory and the calling thread does not wait for work already on `stream`.
+ * Errors: PSS_ERR_INVALID_ARG, PSS_ERR_CAPACITY, PSS_ERR_CUDA.
  */
 pss_status pss_grad_noalloc(const int64_t* table_cardinalities, int32_t num_tables, int32_t dim,
                             int64_t M, int32_t Z, int32_t G, uint64_t seed,

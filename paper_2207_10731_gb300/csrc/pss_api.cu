@@ -503,22 +503,8 @@ pss_status pss_create(const int64_t* cards, int32_t T, int32_t dim, int64_t M, i
     cudaDeviceGetAttribute(&h->sm_count, cudaDevAttrMultiProcessorCount, h->device);
     if (h->sm_count <= 0) h->sm_count = 1;
 
-    // hash parameters from splitmix64(seed)
-    uint64_t s = seed;
-    auto next = [&s]() {
-        s += 0x9e3779b97f4a7c15ULL;
-        uint64_t z = s;
-        z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ULL;
-        z = (z ^ (z >> 27)) * 0x94d049bb133111ebULL;
-        return z ^ (z >> 31);
-    };
-    const uint64_t p61 = (uint64_t(1) << 61) - 1;
-    const uint64_t s1 = next(), s2 = next(), s3 = next(), s4 = next();
     DevParams& dp = h->dp;
-    dp.A = 1 + s1 % (p61 - 1);
-    dp.B0 = s2 % p61;
-    dp.A2 = 1 + s3 % (p61 - 1);
-    dp.B2 = s4 % p61;
+    hash_params_from_seed(seed, &dp);
     dp.smask = 0u;
     dp.G = G;
     dp.M = M;

@@ -19,6 +19,27 @@ struct DevParams {
     uint32_t smask;         // 0x80000000 with signed hashing, else 0 (see pss_device.cuh)
 };
 
+// Hash parameters of a seed (host side, shared by pss_create and
+// pss_grad_noalloc): s1..s4 are the first four splitmix64 outputs (Steele, Lea
+// & Flood 2014) of `seed`, A = 1 + s1 mod (P-1), B0 = s2 mod P for the
+// location hash and A2 = 1 + s3 mod (P-1), B2 = s4 mod P for the sign hash.
+inline void hash_params_from_seed(uint64_t seed, DevParams* p) {
+    const uint64_t p61 = (uint64_t(1) << 61) - 1;
+    uint64_t s = seed;
+    uint64_t out[4];
+    for (int k = 0; k < 4; ++k) {
+        s += 0x9e3779b97f4a7c15ULL;
+        uint64_t z = s;
+        z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ULL;
+        z = (z ^ (z >> 27)) * 0x94d049bb133111ebULL;
+        out[k] = z ^ (z >> 31);
+    }
+    p->A = 1 + out[0] % (p61 - 1);
+    p->B0 = out[1] % p61;
+    p->A2 = 1 + out[2] % (p61 - 1);
+    p->B2 = out[3] % p61;
+}
+
 // Device error word: smallest id position seen out of range, and flag bits.
 struct DevError {
     unsigned long long first_bad;   // ULLONG_MAX when clear

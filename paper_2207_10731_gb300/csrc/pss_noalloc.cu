@@ -70,21 +70,18 @@ bool on_device(const void* p) {
     return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
-// Universal-hash parameters from the seed: the first two splitmix64 outputs
-// (Steele, Lea & Flood 2014), A = 1 + s1 mod (P-1), B0 = s2 mod P.
-void params_from_seed(uint64_t seed, uint64_t* A, uint64_t* B0) {
-    const uint64_t p61 = (uint64_t(1) << 61) - 1;
-    uint64_t s = seed;
-    uint64_t out[2];
-    for (int k = 0; k < 2; ++k) {
-        s += 0x9e3779b97f4a7c15ULL;
-        uint64_t z = s;
-        z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ULL;
-        z = (z ^ (z >> 27)) * 0x94d049bb133111ebULL;
-        out[k] = z ^ (z >> 31);
-    }
-    *A = 1 + out[0] % (p61 - 1);
-    *B0 = out[1] % p61;
+// The table sizes reach the device as kernel arguments, kCardsPerLaunch per
+// launch: no host-to-device copy (a copy from pageable host memory would make
+// the calling thread wait for the work already queued on the stream).
+constexpr int kCardsPerLaunch = 256;
+struct CardsChunk {
+    int64_t v[kCardsPerLaunch];
+    int32_t first, n;
+};
+
+__global__ void k_load_cards(CardsChunk c, int64_t* __restrict__ dst) {
+    pdl_prologue();
+    for (int i = threadIdx.x; i < c.n; i += blockDim.x) dst[c.first + i] = c.v[i];
 }
 
 __global__ void k_error_report(const DevError* err, int64_t* first_bad) {
@@ -132,7 +129,7 @@ extern "C" pss_status pss_grad_noalloc(const int64_t* cards, int32_t T, int32_t 
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
 
     DevParams p{};
-    params_from_seed(seed, &p.A, &p.B0);
+    hash_params_from_seed(seed, &p);
     p.G = G;
     p.M = M;
     p.T = T;
@@ -145,13 +142,20 @@ extern "C" pss_status pss_grad_noalloc(const int64_t* cards, int32_t T, int32_t 
     p.cards = sym.cards;
 
     // The scratch keeps the previous call's contents: clear what must start at
-    // zero (the accumulator and the error word) and load the cardinalities.
+    // zero (the accumulator and the error word) and load the table sizes.
     if (cudaMemsetAsync(sym.accum, 0, sizeof(double) * (size_t)M, st) != cudaSuccess ||
         cudaMemsetAsync(&sym.err->first_bad, 0xff, sizeof(unsigned long long), st) != cudaSuccess ||
-        cudaMemsetAsync(&sym.err->flags, 0, sizeof(unsigned int), st) != cudaSuccess ||
-        cudaMemcpyAsync(sym.cards, cards, sizeof(int64_t) * (size_t)T, cudaMemcpyHostToDevice,
-                        st) != cudaSuccess)
+        cudaMemsetAsync(&sym.err->flags, 0, sizeof(unsigned int), st) != cudaSuccess)
         return PSS_ERR_CUDA;
+    for (int32_t t0 = 0; t0 < T; t0 += kCardsPerLaunch) {
+        CardsChunk c;
+        c.first = t0;
+        c.n = (T - t0) < kCardsPerLaunch ? (T - t0) : kCardsPerLaunch;
+        for (int32_t i = 0; i < c.n; ++i) c.v[i] = cards[t0 + i];
+        if (launch_k(k_load_cards, dim3(1), dim3(kCardsPerLaunch), 0, st, c, sym.cards) !=
+            cudaSuccess)
+            return PSS_ERR_CUDA;
+    }
 
     int sms = 1;
     int dev = 0;

@@ -341,6 +341,61 @@ def test_full_size_step(name):
     h.close()
 
 
+# --------------------------------------------------------------------------
+# scalar-column layouts with several columns per lane (VW = 1, KC = 2 or 4):
+# d > 32 with d, Z or G not a multiple of 4 -- the paper's arbitrary offsets
+# (G = 1) at the Criteo shapes, and the chunk-size study's small chunks
+LAYOUT_CASES = [
+    dict(name="tb", B=2048, G=1),                               # KC = 4, Adagrad
+    dict(name="microbench", B=1024, Z=1, G=1),                  # HashedNet, J = 128
+    dict(name="microbench", B=1024, Z=2, G=1),                  # J = 64
+    dict(name="microbench", B=2048, Z=8),                       # J = 16, 32 ids per round
+    dict(name="multihot", B=512, G=1, bag=("uniform", 0, 40)),  # KC = 2, ragged bags
+]
+
+
+@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("case", LAYOUT_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_scalar_layout_parity(case, path):
+    w = _wl(case)
+    h, o = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    out = gu.host(h.forward(*_batch_cuda(w), w.B)).ravel()
+    ref, bad = o.forward(w.w0, w.indices, w.offsets, w.B)
+    assert bad == -1
+    gu.check_forward(out, ref, _abs_pool(o, w.w0, w), what="scalar-layout forward")
+    del out, ref
+    grads = [("workload", w.grad_out)]
+    if case["name"] == "microbench":
+        # the paper's micro-benchmark loss (all ones) and a signed gradient
+        grads.append(("normal", wl.make_batch(w.cards, w.B, w.d, case.get("bag", ("one",)),
+                                              ("zipf", 1.05), seed=w.seed, batch=0)[2]))
+    for gname, go in grads:
+        h.forward(*_batch_cuda(w), w.B)
+        g = gu.host(h.backward_grad(gu.cuda(go)))
+        A = o.grad(w.indices, w.offsets, w.B, np.abs(go))
+        gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, go), A,
+                      what=f"scalar-layout grad ({gname})")
+        assert h.info()["last_path"] == PATHS[path]
+    # three fused steps with fresh batches, state carried on both sides
+    wcur, Gcur = w.w0.copy(), np.zeros(w.M, dtype=np.float32)
+    h.set_state(gu.cuda(wcur), gu.cuda(Gcur) if w.opt == "adagrad" else None)
+    cfg = wl.CONFIGS[case["name"]]
+    for step in range(3):
+        batch = (w.indices, w.offsets, w.grad_out) if step == 0 else wl.make_batch(
+            w.cards, w.B, w.d, case.get("bag", cfg["bag"]), cfg["ids"], seed=w.seed, batch=step,
+            grad=cfg.get("grad", "normal"))
+        wg, Gg, w2, G2, g32, A = _run_step(w, h, o, wcur, Gcur, batch)
+        if w.opt == "sgd":
+            gu.check_sgd(wg, w2, A, w.lr, what=f"scalar-layout sgd step {step}")
+        else:
+            gu.check_adagrad(wg, Gg, w2, G2, g32, A, w.lr, what=f"scalar-layout adagrad step {step}")
+        wcur, Gcur = w2, (G2 if w.opt == "adagrad" else Gcur)
+        h.set_state(gu.cuda(wcur), gu.cuda(Gcur) if w.opt == "adagrad" else None)
+    assert h.get_error() == (binding.PSS_OK, -1)
+    h.close()
+
+
 def _sub_batch(w, rows):
     """Bags of the given batch rows, all tables, as a smaller batch."""
     rows = np.asarray(rows)
@@ -382,23 +437,15 @@ def test_compression_sweep(logM, path):
         ref, _ = o.forward(w0s, sidx, soff, rows.shape[0])
         absr, _ = o.forward(np.abs(w0s), sidx, soff, rows.shape[0])
     else:
-        # evaluate the oracle on a compact copy of the touched blocks only
+        # the oracle's pooling over a compact copy of the touched blocks: block
+        # k of the copy holds the L elements at the k-th distinct location, and
+        # the locations are remapped to k * L
         locs, _ = o.locations(sidx, soff, rows.shape[0])
-        elems = np.unique((locs[:, None] + np.arange(o.L)[None, :]).ravel())
-        vals = w.w0_at(elems)
-        pos = {int(e): k for k, e in enumerate(elems)}
-        ref = np.zeros(rows.shape[0] * w.T * w.d, np.float64)
-        absr = np.zeros_like(ref)
-        for tt in range(w.T):
-            for bi in range(rows.shape[0]):
-                s = tt * rows.shape[0] + bi
-                for q in range(soff[s], soff[s + 1]):
-                    for j in range(o.J):
-                        base = locs[q * o.J + j]
-                        for z in range(min(w.Z, w.d - j * w.Z)):
-                            v = vals[pos[int(base + z)]]
-                            ref[(bi * w.T + tt) * w.d + j * w.Z + z] += v
-                            absr[(bi * w.T + tt) * w.d + j * w.Z + z] += abs(v)
+        starts, inv = np.unique(locs, return_inverse=True)
+        compact = w.w0_at((starts[:, None] + np.arange(o.L)[None, :]).ravel()).astype(np.float32)
+        clocs = inv.reshape(-1).astype(np.int64) * o.L
+        ref = o.pool(compact, clocs, soff, rows.shape[0], sidx.shape[0])
+        absr = o.pool(np.abs(compact), clocs, soff, rows.shape[0], sidx.shape[0])
     got = gu.host(out[t.from_numpy(rows).cuda()]).ravel()
     gu.check_forward(got, ref, absr, what=f"sweep 2^{logM} forward")
     del out

@@ -4,9 +4,10 @@ It exists for callers that cannot call cudaMalloc -- code embedded in a host
 framework that owns the whole device-memory budget, or latency-critical code
 that cannot accept an allocation's implicit synchronisation.  Its scratch is a
 fixed-size device array inside the library.  These tests call it through the C
-ABI and compare it with the handle-based pss_backward_grad on two calls in a
-row (the second call must not see the first call's leftovers), within the
-gradient tolerance the other parity tests use.
+ABI and compare it with the CPU oracle's gradient on two calls in a row (the
+second call must not see the first call's leftovers), within the gradient
+tolerance the other parity tests use, and with the handle-based
+pss_backward_grad on the same inputs.
 """
 import ctypes
 
@@ -30,25 +31,31 @@ def _call(lib, w, indices, offsets, grad_out, grad, first_bad, stream):
                                 ctypes.c_void_p(int(stream.cuda_stream)))
 
 
-@pytest.mark.parametrize("name,B", [("kaggle", 2048), ("tb", 4096), ("multihot", 1024)])
-def test_noalloc_gradient_matches_handle_gradient_two_calls(name, B):
+# 300 tables: the table sizes reach the device in two launches of 256
+@pytest.mark.parametrize("name,B,over", [("kaggle", 2048, {}), ("tb", 4096, {}),
+                                         ("multihot", 1024, {}), ("tiny", 64, {"T": 300})],
+                         ids=["kaggle", "tb", "multihot", "tiny-300-tables"])
+def test_noalloc_gradient_matches_oracle_two_calls(name, B, over):
     t = gu.torch()
     lib = binding.load_library()
     stream = t.cuda.current_stream()
     for batch in (0, 1):
-        w = wl.make_workload(name, B=B, batch=batch)
+        w = wl.make_workload(name, B=B, batch=batch, **over)
         assert w.M <= MAX_M
         h, o = gu.make_pair(w)
         idx, off, go = gu.cuda(w.indices), gu.cuda(w.offsets), gu.cuda(w.grad_out)
         h.forward(idx, off, w.B)
-        g_ref = gu.host(h.backward_grad(go)).astype(np.float64)
+        g_handle = gu.host(h.backward_grad(go)).astype(np.float64)
         h.close()
         grad = t.full((w.M,), float("nan"), dtype=t.float32, device="cuda")
         first_bad = t.zeros(1, dtype=t.int64, device="cuda")
         assert _call(lib, w, idx, off, go, grad, first_bad, stream) == binding.PSS_OK
         t.cuda.synchronize()
+        g_ref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
         A = o.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
-        gu.check_grad(gu.host(grad), g_ref, A, what=f"noalloc {name} batch {batch}")
+        g = gu.host(grad)
+        gu.check_grad(g, g_ref, A, what=f"noalloc {name} batch {batch} vs oracle")
+        gu.check_grad(g, g_handle, 2 * A, what=f"noalloc {name} batch {batch} vs handle")
         assert int(first_bad.item()) == -1
 
 
