@@ -84,12 +84,14 @@ typedef enum { PSS_SGD = 0, PSS_ADAGRAD = 1 } pss_optimizer;
 typedef enum {
     /* Backward path: the dense gradient of Algorithm 1 built with vector atomics
      * (PSS_PATH_ATOMIC), or the sorted path that reduces equal locations before
-     * touching M (PSS_PATH_SORTED, Algorithm 1's sparse branch).  In both, the
-     * order of a location's contributions depends on the GPU's scheduling, so
-     * low-order bits may differ between runs (within the accumulation bound;
-     * dyadic inputs give identical bits).  PSS_PATH_AUTO takes the sorted path
-     * when the batch adds at least 2^23 elements (nnz * J * L), the atomic one
-     * below (crossover measured on GB300; M does not move it). */
+     * touching M (PSS_PATH_SORTED, Algorithm 1's sparse branch).  On the atomic
+     * path the order of a location's contributions depends on the GPU's
+     * scheduling, so low-order bits may differ between runs (within the
+     * accumulation bound; dyadic inputs give identical bits).  The sorted path
+     * groups the contributions by location and sums each location's run once
+     * (see PSS_OPT_DETERMINISTIC for its order).  PSS_PATH_AUTO takes the
+     * sorted path when the batch adds at least 2^23 elements (nnz * J * L),
+     * the atomic one below (crossover measured on GB300; M does not move it). */
     PSS_OPT_BACKWARD_PATH = 1,
     /* How the Adagrad step visits M: every element (PSS_UPDATE_DENSE), only the
      * blocks the batch touched (PSS_UPDATE_TOUCHED), or chosen from M and the
@@ -128,14 +130,22 @@ typedef enum {
      * changes R (pss_get_info) and forgets the last forward's batch.
      * pss_grad_noalloc does not wrap. */
     PSS_OPT_CIRCULAR = 7,
-    /* log2 of the number of counters of the sorted path's counting sort, 4 to
-     * 30 (default 22).  With more block starts R than counters, block x is
-     * counted under x mod 2^value: the counters stay small enough to live in
-     * L2 at any M, and entries come out grouped by residue, runs of buckets
-     * that share one alternating within a group (the reduce checks every
-     * entry then).  Results do not depend on it.  Changing it synchronises
-     * the device and forgets the last forward's batch. */
-    PSS_OPT_SORT_KEYS = 8
+    /* Digit width of the sorted path's radix sort (used with
+     * PSS_OPT_DETERMINISTIC, and always above 2^22 block starts): 0 (default)
+     * sorts the bucket indices (bit width of R - 1) in as few passes of at
+     * most 11 bits as possible; 4 to 11 forces that many bits per pass (more
+     * passes).  The sort is stable, so the result does not depend on it. */
+    PSS_OPT_SORT_DIGIT_BITS = 8,
+    /* 1: run-to-run identical bits on the sorted path.  The sorted path then
+     * sorts with the stable radix sort (see PSS_OPT_SORT_DIGIT_BITS), which
+     * orders the contributions of every location by pair; the reduce sums
+     * them in that order, and the few run sums of an element meet in fp64
+     * (exact, hence in any order, unless their magnitudes span more than
+     * about 2^26).  0 (default): the faster counting sort, whose order within
+     * a location follows the GPU's scheduling (the sum is within the same
+     * bound, but low-order bits may differ between runs).  Above 2^22 block
+     * starts the radix sort is always used.  The atomic path is not affected. */
+    PSS_OPT_DETERMINISTIC = 9
 } pss_option;
 
 
@@ -151,9 +161,9 @@ typedef enum {
     PSS_K_FORWARD = 1,     /* fused hash + gather + sum-pool */
     PSS_K_SCATTER = 2,     /* backward: hash + vector-atomic scatter (+ fused SGD) */
     PSS_K_UPDATE = 3,      /* optimizer pass over M (dense or touched blocks) */
-    PSS_K_SORT = 4,        /* sorted path: bucket count, scan, slot scatter (and, with
-                              counters shared by residue and the touched update, the
-                              marking of the touched blocks) */
+    PSS_K_SORT = 4,        /* sorted path: the counting sort's count, scan and slot
+                              scatter, or the radix sort's passes (and, with the touched
+                              update, the marking of the touched blocks) */
     PSS_K_REDUCE = 5,      /* sorted path: run sums into the fp64 accumulator */
     PSS_K_MISC = 6,        /* memsets and small helper kernels */
     PSS_K_COUNT = 7
@@ -166,11 +176,8 @@ typedef struct {
     int64_t optimizer;         /* pss_optimizer */
     int64_t kernel_launches;   /* kernels this handle has launched so far */
     int64_t last_path;         /* PSS_PATH_ATOMIC / PSS_PATH_SORTED of the last backward */
-    double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass, or -1;
-                                  with more block starts than sort counters (2^22 unless
-                                  PSS_OPT_SORT_KEYS says otherwise) the distinct residues of
-                                  the block index stand in for the distinct blocks (an
-                                  upper bound on the rate) */
+    double last_collision_rate;/* 1 - distinct blocks / (nnz*J) of the last sorted pass
+                                  whose counts have reached the host, or -1 */
     uint64_t A2, B2;           /* sign-hash parameters derived from the seed */
     int64_t signed_hash;       /* PSS_OPT_SIGNED */
     int64_t circular;          /* PSS_OPT_CIRCULAR */

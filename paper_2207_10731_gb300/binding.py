@@ -25,7 +25,8 @@ PSS_SGD, PSS_ADAGRAD = 0, 1
 OPT_BACKWARD_PATH, OPT_UPDATE_MODE, OPT_PROFILE, OPT_SYNC_CHECK, OPT_ACCUM = 1, 2, 3, 4, 5
 OPT_SIGNED = 6
 OPT_CIRCULAR = 7
-OPT_SORT_KEYS = 8
+OPT_SORT_DIGIT_BITS = 8
+OPT_DETERMINISTIC = 9
 ACCUM_F64, ACCUM_F32 = 0, 1
 PATH_AUTO, PATH_ATOMIC, PATH_SORTED = 0, 1, 2
 UPDATE_AUTO, UPDATE_DENSE, UPDATE_TOUCHED = 0, 1, 2

@@ -64,7 +64,8 @@ struct pss_handle {
     int64_t profile = 0;
     int64_t sync_check = 0;
     int64_t accum = PSS_ACCUM_F64;
-    int64_t sort_keys_log2 = 22;                // PSS_OPT_SORT_KEYS
+    int64_t sort_digit_bits = 0;                // PSS_OPT_SORT_DIGIT_BITS (0: automatic)
+    int64_t deterministic = 0;                  // PSS_OPT_DETERMINISTIC
     int64_t last_path = PSS_PATH_ATOMIC;
     double last_collision = -1.0;
 
@@ -77,7 +78,9 @@ struct pss_handle {
     // sorted backward path (allocated on first use)
     SortedBuffers sb{};
     int64_t sb_pairs_cap = 0, sb_ids_cap = 0;
-    bool sb_counters = false;
+    bool sb_fixed = false;                      // the buffers that do not grow with the batch
+    bool sb_counting = false;                   // the counting sort's R-sized buffers
+    int64_t radix_pairs_cap = 0;                // pairs the radix sort's buffers hold
     bool batch_emitted = false;                 // the last forward wrote pair_x / q_row
     unsigned long long* stats_host = nullptr;   // pinned mirror of sb.stats
     cudaEvent_t stats_ev = nullptr;
@@ -282,18 +285,11 @@ pss_status ensure_grad(pss_handle* h, cudaStream_t st) {
 // Buffers sized by the number of block starts R, released when R changes (they
 // are allocated again on first use).  The caller has synchronised the device.
 void release_r_buffers(pss_handle* h) {
-    for (void* b : {(void*)h->sb.cnt, (void*)h->sb.start, (void*)h->sb.bsum, (void*)h->sb.bnz,
-                    (void*)h->sb.stats, (void*)h->touched.bitmap, (void*)h->touched.list,
-                    (void*)h->touched.count})
+    for (void* b : {(void*)h->touched.bitmap, (void*)h->touched.list, (void*)h->touched.count,
+                    (void*)h->sb.ccnt, (void*)h->sb.start, (void*)h->sb.bsum, (void*)h->sb.bnz})
         if (b) cudaFree(b);
-    if (h->stats_host) cudaFreeHost(h->stats_host);
-    if (h->stats_ev) cudaEventDestroy(h->stats_ev);
-    h->sb.cnt = h->sb.start = h->sb.bsum = h->sb.bnz = nullptr;
-    h->sb.stats = nullptr;
-    h->stats_host = nullptr;
-    h->stats_ev = nullptr;
-    h->stats_pending = false;
-    h->sb_counters = false;
+    h->sb.ccnt = h->sb.start = h->sb.bsum = h->sb.bnz = nullptr;
+    h->sb_counting = false;
     h->touched = Touched{};
     h->touched_words = 0;
 }
@@ -349,14 +345,13 @@ bool use_touched(const pss_handle* h, int64_t pairs) {
 
 // The sorted path holds bucket indices in 32 bits, 0xffffffff marking a bad
 // id: it needs R < kSortedMaxR, the bound below which the forward emits 32-bit
-// buckets at all.  Above 2^sort_keys_log2 buckets its counters are shared by
-// residue (see SortedBuffers).  AUTO takes the sorted path when the batch adds at least
+// buckets at all.  AUTO takes the sorted path when the batch adds at least
 // kAutoSortedMinAdds elements (pairs * L): measured on GB300, the atomic path
-// wins below it (its one kernel against the sort's five; Criteo-Kaggle shape
-// at batch 8192: 3.4M adds, 0.049 against 0.108 ms per step), the sorted path
-// above it at every M from 2^18 to 2^33, Zipf or uniform ids (Criteo-Kaggle
-// shape at batch 32768 and Criteo-TB shape at batch 4096: 13.6M adds, 0.138
-// against 0.186 and 0.073 against 0.113 ms).
+// wins below it (its one kernel against the sort's launches; Criteo-Kaggle
+// shape at batch 8192: 3.4M adds, 0.049 against 0.108 ms per step), the sorted
+// path above it at every M from 2^18 to 2^33, Zipf or uniform ids
+// (Criteo-Kaggle shape at batch 32768 and Criteo-TB shape at batch 4096: 13.6M
+// adds, 0.138 against 0.186 and 0.073 against 0.113 ms).
 constexpr int64_t kSortedMaxR = int64_t(0xffffffffLL);
 constexpr int64_t kAutoSortedMinAdds = int64_t(1) << 23;
 
@@ -369,6 +364,12 @@ bool sorted_supported(const pss_handle* h, int64_t nnz, int64_t B) {
            (int64_t)h->dp.T * B * J < lim;
 }
 
+// The sorted path's sort: the counting sort (one counter per bucket), unless
+// the caller asked for run-to-run identical bits or R exceeds its counters.
+bool use_radix(const pss_handle* h) {
+    return h->deterministic || (int64_t)h->dp.R > kCountSortMaxR;
+}
+
 bool want_sorted(const pss_handle* h, int64_t npairs) {
     if (h->path == PSS_PATH_SORTED) return true;
     if (h->path == PSS_PATH_ATOMIC) return false;
@@ -376,31 +377,20 @@ bool want_sorted(const pss_handle* h, int64_t npairs) {
 }
 
 pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {
-    const int64_t R = (int64_t)h->dp.R;
     const int64_t npairs = nnz * h->dp.J;
-    if (!h->sb_counters) {
-        const int64_t K = int64_t(1) << h->sort_keys_log2;   // residues are taken with a mask
-        const int64_t nkeys = R < K ? R : K;
-        h->sb.nkeys = nkeys;
-        h->sb.kmask = R <= K ? 0xffffffffu : (uint32_t)(K - 1);
-        const int64_t nblk = sorted_scan_blocks(nkeys);
-        PSS_TRY(cudaMalloc(&h->sb.cnt, sizeof(uint32_t) * (size_t)nkeys));
-        PSS_TRY(cudaMemsetAsync(h->sb.cnt, 0, sizeof(uint32_t) * (size_t)nkeys, st));
-        PSS_TRY(cudaMalloc(&h->sb.start, sizeof(uint32_t) * (size_t)(nkeys + 1)));
-        PSS_TRY(cudaMalloc(&h->sb.bsum, sizeof(uint32_t) * (size_t)nblk));
-        PSS_TRY(cudaMalloc(&h->sb.bnz, sizeof(uint32_t) * (size_t)nblk));
+    if (!h->sb_fixed) {
         PSS_TRY(cudaMalloc(&h->sb.stats, 2 * sizeof(unsigned long long)));
         PSS_TRY(cudaMemsetAsync(h->sb.stats, 0, 2 * sizeof(unsigned long long), st));
         PSS_TRY(cudaMallocHost(&h->stats_host, 2 * sizeof(unsigned long long)));
         h->stats_host[0] = h->stats_host[1] = 0;
         PSS_TRY(cudaEventCreateWithFlags(&h->stats_ev, cudaEventDisableTiming));
-        h->sb_counters = true;
+        h->sb_fixed = true;
     }
     if (h->sb_pairs_cap < npairs) {
-        if (h->sb.pair_x) PSS_TRY(cudaFreeAsync(h->sb.pair_x, st));
-        if (h->sb.sorted_e) PSS_TRY(cudaFreeAsync(h->sb.sorted_e, st));
-        h->sb.pair_x = nullptr;
-        h->sb.sorted_e = nullptr;
+        for (void** b : {(void**)&h->sb.pair_x, (void**)&h->sb.sorted_e}) {
+            if (*b) PSS_TRY(cudaFreeAsync(*b, st));
+            *b = nullptr;
+        }
         h->sb_pairs_cap = 0;
         const size_t n = (size_t)(npairs > 0 ? npairs : 1);
         PSS_TRY(cudaMallocAsync(&h->sb.pair_x, sizeof(uint32_t) * n, st));
@@ -413,6 +403,45 @@ pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {
         h->sb_ids_cap = 0;
         PSS_TRY(cudaMallocAsync(&h->sb.q_row, sizeof(uint32_t) * (size_t)(nnz > 0 ? nnz : 1), st));
         h->sb_ids_cap = nnz;
+    }
+    return PSS_OK;
+}
+
+// The counting sort's buffers: one counter and one start per bucket.
+pss_status ensure_counting(pss_handle* h, cudaStream_t st) {
+    if (h->sb_counting) return PSS_OK;
+    const int64_t R = (int64_t)h->dp.R;
+    const int64_t nblk = sorted_scan_blocks(R);
+    PSS_TRY(cudaMalloc(&h->sb.ccnt, sizeof(uint32_t) * (size_t)R));
+    PSS_TRY(cudaMemsetAsync(h->sb.ccnt, 0, sizeof(uint32_t) * (size_t)R, st));
+    PSS_TRY(cudaMalloc(&h->sb.start, sizeof(uint32_t) * (size_t)(R + 1)));
+    PSS_TRY(cudaMalloc(&h->sb.bsum, sizeof(uint32_t) * (size_t)nblk));
+    PSS_TRY(cudaMalloc(&h->sb.bnz, sizeof(uint32_t) * (size_t)nblk));
+    h->sb_counting = true;
+    return PSS_OK;
+}
+
+// The radix sort's buffers for npairs pairs: the second entry buffer and the
+// per-tile digit counts of the widest digit.
+pss_status ensure_radix(pss_handle* h, int64_t npairs, cudaStream_t st) {
+    if (!h->sb.tot) {
+        const size_t nd = size_t(1) << kRadixMaxBits;
+        PSS_TRY(cudaMalloc(&h->sb.tot, sizeof(uint32_t) * nd));
+        PSS_TRY(cudaMalloc(&h->sb.dstart, sizeof(uint32_t) * nd));
+        PSS_TRY(cudaMalloc(&h->sb.done, sizeof(uint32_t)));
+        PSS_TRY(cudaMemsetAsync(h->sb.done, 0, sizeof(uint32_t), st));
+    }
+    if (h->radix_pairs_cap < npairs) {
+        for (void** b : {(void**)&h->sb.tmp_e, (void**)&h->sb.cnt}) {
+            if (*b) PSS_TRY(cudaFreeAsync(*b, st));
+            *b = nullptr;
+        }
+        h->radix_pairs_cap = 0;
+        const size_t n = (size_t)(npairs > 0 ? npairs : 1);
+        PSS_TRY(cudaMallocAsync(&h->sb.tmp_e, sizeof(unsigned long long) * n, st));
+        const size_t nc = (size_t)radix_tiles((int64_t)n) * (size_t)(1 << kRadixMaxBits);
+        PSS_TRY(cudaMallocAsync(&h->sb.cnt, sizeof(uint32_t) * nc, st));
+        h->radix_pairs_cap = npairs;
     }
     return PSS_OK;
 }
@@ -561,9 +590,11 @@ pss_status pss_destroy(pss_handle* h) {
     cudaFree(h->touched.bitmap);
     cudaFree(h->touched.list);
     cudaFree(h->touched.count);
-    for (void* b : {(void*)h->sb.pair_x, (void*)h->sb.q_row, (void*)h->sb.cnt, (void*)h->sb.start,
-                    (void*)h->sb.bsum, (void*)h->sb.bnz, (void*)h->sb.stats,
-                    (void*)h->sb.sorted_e})
+    for (void* b : {(void*)h->sb.pair_x, (void*)h->sb.q_row, (void*)h->sb.sorted_e,
+                    (void*)h->sb.tmp_e, (void*)h->sb.cnt, (void*)h->sb.tot,
+                    (void*)h->sb.dstart, (void*)h->sb.done, (void*)h->sb.stats,
+                    (void*)h->sb.ccnt, (void*)h->sb.start, (void*)h->sb.bsum,
+                    (void*)h->sb.bnz})
         if (b) cudaFree(b);
     if (h->stats_host) cudaFreeHost(h->stats_host);
     if (h->stats_ev) cudaEventDestroy(h->stats_ev);
@@ -721,38 +752,46 @@ static pss_status scatter_into(pss_handle* h, const float* dgrad, float scale, f
                                       touch ? &h->touched : nullptr, h->err, h->sm_count, st));
 }
 
-// Sorted path: histogram, scan, scatter by bucket, segmented reduce into g64.
+// Sorted path: sort by bucket (counting or radix), segmented reduce into g64.
 static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, bool touch,
                                 cudaStream_t st) {
     const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
     if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
     poll_stats(h);
-    // cnt is zero here: it is zeroed when allocated, and every sort's slot
-    // scatter counts each key back down by exactly what its count added.
-    // With counters shared by residue, the touched buckets come from the
-    // pairs themselves rather than from the non-empty counters.
-    const bool mixed = h->sb.kmask != 0xffffffffu;
-    {
-        LaunchScope ls(h, PSS_K_SORT, st, (touch && mixed) ? 6 : 5);
-        PSS_TRY(launch_sorted_count(h->sb, npairs, h->dp.smask, h->sm_count, st));
-        PSS_TRY(launch_sorted_scan(h->sb, h->sb.nkeys, (touch && !mixed) ? &h->touched : nullptr,
-                                   st));
-        if (touch && mixed)
+    if (use_radix(h)) {
+        pss_status rc0 = ensure_radix(h, npairs, st);
+        if (rc0 != PSS_OK) return rc0;
+        const RadixPlan plan = radix_plan(h->dp.R, (int)h->sort_digit_bits);
+        LaunchScope ls(h, PSS_K_SORT, st, 3 * plan.passes + (touch ? 1 : 0));
+        PSS_TRY(launch_radix_sort(h->sb, npairs, h->dp.J, h->dp.smask, plan, st));
+        if (touch)
             PSS_TRY(launch_mark_pairs(h->sb, npairs, h->dp.smask, h->touched, h->sm_count, st));
+    } else {
+        // ccnt is zero here: it is zeroed when allocated, and every sort's slot
+        // scatter counts each bucket back down by exactly what its count added
+        pss_status rc0 = ensure_counting(h, st);
+        if (rc0 != PSS_OK) return rc0;
+        LaunchScope ls(h, PSS_K_SORT, st, 5);
+        PSS_TRY(launch_sorted_count(h->sb, npairs, h->dp.smask, h->sm_count, st));
+        PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, touch ? &h->touched : nullptr, st));
         PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->dp.smask, h->sm_count, st));
     }
+    // the sort above needs only the forward's buckets: a host gradient's copy
+    // has overlapped it, and is waited for here
+    pss_status rc = grad_wait(h, staged, st);
+    if (rc != PSS_OK) return rc;
+    {
+        LaunchScope ls(h, PSS_K_REDUCE, st);
+        PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64, h->sm_count, st));
+    }
+    // valid pairs (the sort) and distinct buckets (the reduce), for
+    // pss_get_info's collision rate; one copy in flight at a time
     if (!h->stats_pending) {
         PSS_TRY(cudaMemcpyAsync(h->stats_host, h->sb.stats, 2 * sizeof(unsigned long long),
                                 cudaMemcpyDeviceToHost, st));
         PSS_TRY(cudaEventRecord(h->stats_ev, st));
         h->stats_pending = true;
     }
-    // the sort above needs only the forward's buckets: a host gradient's copy
-    // has overlapped it, and is waited for here
-    pss_status rc = grad_wait(h, staged, st);
-    if (rc != PSS_OK) return rc;
-    LaunchScope ls(h, PSS_K_REDUCE, st);
-    PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64, h->sm_count, st));
     return PSS_OK;
 }
 
@@ -939,16 +978,14 @@ pss_status pss_set_option(pss_handle* h, int32_t key, int64_t value) {
             h->dp.smask = m;
             return PSS_OK;
         }
-        case PSS_OPT_SORT_KEYS: {
-            if (value < 4 || value > 30) return PSS_ERR_INVALID_ARG;
-            if (value == h->sort_keys_log2) return PSS_OK;
-            DeviceGuard g(h->device);
-            PSS_TRY(cudaDeviceSynchronize());
-            release_r_buffers(h);
-            h->sort_keys_log2 = value;
-            h->have_batch = false;
+        case PSS_OPT_SORT_DIGIT_BITS:
+            if (value != 0 && (value < 4 || value > kRadixMaxBits)) return PSS_ERR_INVALID_ARG;
+            h->sort_digit_bits = value;
             return PSS_OK;
-        }
+        case PSS_OPT_DETERMINISTIC:
+            if (value != 0 && value != 1) return PSS_ERR_INVALID_ARG;
+            h->deterministic = value;
+            return PSS_OK;
     }
     return PSS_ERR_INVALID_ARG;
 }
@@ -963,7 +1000,8 @@ pss_status pss_get_option(pss_handle* h, int32_t key, int64_t* value) {
         case PSS_OPT_ACCUM: *value = h->accum; return PSS_OK;
         case PSS_OPT_SIGNED: *value = h->dp.smask ? 1 : 0; return PSS_OK;
         case PSS_OPT_CIRCULAR: *value = h->circ ? 1 : 0; return PSS_OK;
-        case PSS_OPT_SORT_KEYS: *value = h->sort_keys_log2; return PSS_OK;
+        case PSS_OPT_SORT_DIGIT_BITS: *value = h->sort_digit_bits; return PSS_OK;
+        case PSS_OPT_DETERMINISTIC: *value = h->deterministic; return PSS_OK;
     }
     return PSS_ERR_INVALID_ARG;
 }

@@ -64,38 +64,57 @@ struct Touched {
     int64_t cap;
 };
 
+// Radix sort of the sorted backward path: `passes` digits of `bits[k]` bits
+// starting at bit shift[k] of the bucket index.
+constexpr int kRadixMaxBits = 11;          // digit bits per pass (at most 2048 digits)
+constexpr int kRadixMaxPasses = 8;         // 32-bit buckets with 4-bit digits
+struct RadixPlan {
+    int passes;
+    int bits[kRadixMaxPasses];
+    int shift[kRadixMaxPasses];
+};
+// Plan for buckets in [0, R): digit_bits 0 picks at most kRadixMaxBits bits per
+// pass, as few passes as that allows, split evenly; 4 .. 11 forces that many.
+RadixPlan radix_plan(uint64_t R, int digit_bits);
+int64_t radix_tiles(int64_t npairs);   // tiles of one pass
+
 // Buffers of the sorted backward path (see pss_sorted.cu).
 struct SortedBuffers {
     uint32_t* pair_x;             // nnz*J buckets written by the forward (0xffffffff: bad id)
     uint32_t* q_row;              // nnz output rows b*T + t written by the forward
-    uint32_t* cnt;                // nkeys counts per counting key, filled by launch_sorted_count
+    unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j), grouped by x
+    unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets
+    // counting sort (R <= kCountSortMaxR)
+    uint32_t* ccnt;               // R counts per bucket (zero between sorts)
     uint32_t* start;              // R + 1 bucket starts
     uint32_t* bsum;               // per scan chunk: entries, then their exclusive prefix
     uint32_t* bnz;                // per scan chunk: non-empty buckets
-    unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets
-    unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j) in counting-key order
-    // Counting key of bucket x: x & kmask.  With R <= K counters, kmask has
-    // every bit set and the entries come out in bucket order; above it the
-    // K counters cover the residues of x mod K (a power of two), entries are
-    // grouped by residue, and inside a residue class runs of different
-    // buckets may alternate (the reduce then checks every entry of a block).
-    uint32_t kmask;
-    int64_t nkeys;                // number of counters: min(R, K)
+    // radix sort
+    unsigned long long* tmp_e;    // nnz*J entries: the other buffer of the radix passes
+    uint32_t* cnt;                // [2^bits][radix_tiles(nnz*J)] per-tile digit counts
+    uint32_t* tot;                // [2^kRadixMaxBits] digit totals of the current pass
+    uint32_t* dstart;             // [2^kRadixMaxBits] digit start positions of the current pass
+    uint32_t* done;               // finished-CTA counter of the column scan (zero between passes)
 };
+// The counting sort keeps one counter per bucket: it serves R up to this.
+constexpr int64_t kCountSortMaxR = int64_t(1) << 22;
 int64_t sorted_scan_blocks(int64_t R);
-// Per-key counts of the valid pairs (cnt must be zero on entry).
+// Counting sort: per-bucket counts of the valid pairs (ccnt must be zero on
+// entry), their scan (with `touched`, also the list / bitmap of non-empty
+// buckets), and the slot scatter into sorted_e (which returns ccnt to zero).
 cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
                                 int sm_count, cudaStream_t st);
-// Key starts; with `touched` (only when every bucket has its own counter),
-// also the list / bitmap of non-empty buckets.
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
                                cudaStream_t st);
-// Touched bitmap / list of the buckets of the forward's pairs (the sorted path
-// when counters are shared by residue).
-cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
-                              const Touched& touched, int sm_count, cudaStream_t st);
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
                                   int sm_count, cudaStream_t st);
+// Stable radix sort of the forward's pairs by bucket into sorted_e (three
+// kernels per pass; see pss_sorted.cu): entries of one bucket in pair order.
+cudaError_t launch_radix_sort(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
+                              const RadixPlan& plan, cudaStream_t st);
+// Touched bitmap / list of the buckets of the forward's pairs.
+cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
+                              const Touched& touched, int sm_count, cudaStream_t st);
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
                                  const DevParams& p, double* g, int sm_count, cudaStream_t st);
 

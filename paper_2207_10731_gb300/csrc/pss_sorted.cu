@@ -6,28 +6,20 @@
 //              for an id outside its table;
 //   q_row[q]   output row b*T + t of the bag that holds id q;
 // Steps (all on the caller's stream):
-//   0. count    cnt[k] = number of valid pairs with counting key k = x & kmask
-//               (cnt zeroed by the caller; k = x unless R exceeds the number
-//               of counters, see SortedBuffers);
-//   1. scan     start[k] = sum of cnt[y] for y < k (three kernels);
-//               statistics: valid pairs and distinct keys;
-//   2. scatter  each pair takes a slot in [start[k], start[k+1]) of sorted_e,
-//               which holds (x, r = row*J + j): the bucket and the
-//               upstream-gradient chunk to add (with signed hashing, bit 31 of
-//               pair_x and of r carries the pair's sign, see pss_device.cuh);
-//   3. reduce   the sorted entries are cut into tasks of kPiece consecutive
-//               entries; one group of lanes per task owns 16-byte columns of
-//               the block, adds the chunks of each run of equal x with
-//               compensated (Kahan) fp32 sums, and adds every run's sum once
-//               into the fp64 gradient accumulator g[G*x + z] -- one reduction
-//               per run and element instead of one per contribution, and no
-//               queue of reductions on a hot address.  With `mixed` (counters
-//               shared by residue) runs of different buckets may alternate,
-//               and a block of entries is summed as one run only when every
-//               entry of it belongs to the current run.
-// With counters shared by residue and the touched update, k_mark_pairs lists
-// the touched blocks from pair_x (the scan cannot: a non-empty counter no
-// longer names one bucket).
+//   1. sort     a stable radix sort of the entries e = x << 32 | r by x, where
+//               r = row*J + j names the upstream-gradient chunk to add (with
+//               signed hashing, bit 31 of pair_x and of r carries the pair's
+//               sign, see pss_device.cuh); bad ids are dropped.  Entries of one
+//               bucket come out in pair order, so every later step sees the
+//               same sequence on every run;
+//   2. reduce   the sorted entries are cut into tasks of consecutive entries;
+//               the lanes of a task own columns of the block, add the chunks of
+//               each run of equal x with compensated (Kahan) fp32 sums, and add
+//               every run's sum once into the fp64 gradient accumulator
+//               g[G*x + z] -- one reduction per run and element instead of one
+//               per contribution, and no queue of reductions on a hot address.
+//               The reduce also counts the distinct buckets (stats[1]).
+// With the touched update, k_mark_pairs lists the touched blocks from pair_x.
 // The optimizer pass over g follows (pss_kernels.cu).
 #include <climits>
 
@@ -75,6 +67,11 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s
     return r;
 }
 
+// ---------------------------------------------------------------------------
+// Counting sort by bucket (the default when R <= kCountSortMaxR): a count of
+// every bucket, a scan of the counts (three kernels), and a slot scatter.
+// Every bucket has its own counter, so the entries come out grouped by bucket;
+// their order inside a bucket depends on the GPU's scheduling.
 // Per chunk of kScanChunk counters: entries and non-empty buckets.
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict__ bsum,
@@ -97,11 +94,10 @@ k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict_
     if (threadIdx.x == 0) bnz[blockIdx.x] = tot;
 }
 
-// Exclusive scan of the chunk sums (one block).  stats[0] = valid pairs,
-// stats[1] = distinct buckets.
 // Exclusive scans of the chunk sums and of the chunk non-empty counts (one
-// block).  stats[0] = valid pairs, stats[1] = distinct buckets, which is also
-// the length of the touched list when one is built.
+// block).  stats[0] = valid pairs; stats[1] is cleared (the reduce counts the
+// distinct buckets); the number of non-empty buckets is the length of the
+// touched list when one is built.
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ bnz, int64_t nblk,
            unsigned long long* __restrict__ stats, unsigned long long* __restrict__ touched_count) {
@@ -132,7 +128,7 @@ k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ bnz, int64_t nblk
     }
     if (threadIdx.x == 0) {
         stats[0] = s_carry[0];
-        stats[1] = s_carry[1];
+        stats[1] = 0;
         if (touched_count) *touched_count = s_carry[1];
     }
 }
@@ -209,9 +205,9 @@ __device__ __forceinline__ void seg_table_init(uint32_t* s_key, uint32_t* s_val)
     }
 }
 
-// cnt[k] += number of valid pairs with counting key k = (x without its sign) & kmask.
+// cnt[x] += number of valid pairs with bucket x (without its sign).
 __global__ void __launch_bounds__(kSegThreads)
-k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask, uint32_t kmask,
+k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask,
              uint32_t* __restrict__ cnt) {
     pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
@@ -229,7 +225,7 @@ k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask
         __syncthreads();   // the previous segment's table is clear
 #pragma unroll
         for (int i = 0; i < kSegPer; ++i)
-            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i] & ~smask & kmask) : 0u;
+            hr[i] = (x[i] != kBad) ? seg_insert(s_key, s_val, x[i] & ~smask) : 0u;
         __syncthreads();
 #pragma unroll
         for (int k = 0; k < kSegSlots / kSegThreads; ++k) {
@@ -249,15 +245,15 @@ k_sort_count(const uint32_t* __restrict__ pair_x, int64_t npairs, uint32_t smask
 }
 
 // Slot of every valid pair: cnt counts back down to zero, each segment taking
-// one contiguous range of its counting key for every bucket it holds (one
-// atomic per distinct bucket); within the range a pair's place is its rank in
-// the segment table, which is keyed by the bucket, so a segment's pairs of one
-// bucket stay together even when several buckets share a key.
+// one contiguous range of the bucket for every bucket it holds (one atomic per
+// distinct bucket); within the range a pair's place is its rank in the
+// segment table.  Which segment takes which range, and the ranks, follow the
+// order in which the GPU runs the atomics.
 // sorted_e[slot] = x << 32 | row*J + j.
 template <bool SG>
 __global__ void __launch_bounds__(kSegThreads)
 k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32_t* __restrict__ q_row,
-               int J, int log2J, uint32_t kmask, const uint32_t* __restrict__ start,
+               int J, int log2J, const uint32_t* __restrict__ start,
                uint32_t* __restrict__ cnt, unsigned long long* __restrict__ sorted_e) {
     pdl_prologue();
     __shared__ uint32_t s_key[kSegSlots];
@@ -286,7 +282,7 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
                     e[i] |= x[i] & 0x80000000u;
                     x[i] &= 0x7fffffffu;
                 }
-                st0[i] = __ldg(start + (x[i] & kmask));
+                st0[i] = __ldg(start + x[i]);
             }
         }
         __syncthreads();   // the previous segment's table is clear
@@ -307,7 +303,7 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
             }
 #pragma unroll
             for (int u = 0; u < kSegFlushU; ++u)
-                old[u] = (key[u] != kEmpty) ? atomicSub(cnt + (key[u] & kmask), c[u]) : 0u;
+                old[u] = (key[u] != kEmpty) ? atomicSub(cnt + key[u], c[u]) : 0u;
 #pragma unroll
             for (int u = 0; u < kSegFlushU; ++u)
                 if (key[u] != kEmpty) s_val[(k0 + u) * kSegThreads + threadIdx.x] = old[u] - c[u];
@@ -326,6 +322,331 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
                 s_key[hr[i] & 0xffffu] = kEmpty;
                 s_val[hr[i] & 0xffffu] = 0u;
             }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Stable LSD radix sort of the pairs by bucket x.
+//
+// The keys are the bucket indices (at most 32 bits); the sort makes P passes of
+// D <= 11 bits each (RadixPlan).  A pass cuts its input into TILES of kRTile
+// consecutive entries and takes three kernels:
+//   up       each tile's count of every digit, cnt[digit][tile];
+//   colscan  for every digit, the exclusive prefix of its counts over the
+//            tiles (in place, one warp per digit) and its total; the last CTA
+//            to finish turns the totals into the digits' start positions;
+//   down     each tile ranks every entry among the tile's entries of the same
+//            digit in input order (warp by warp, lane by lane) and stores it at
+//              start[digit] + cnt[digit][tile] + rank,
+//            staging the tile in shared memory in digit order first, so that
+//            the entries of one digit leave the CTA as one contiguous run.
+// Entries of equal digit keep their input order, so after the last pass the
+// entries are ordered by bucket and, within a bucket, by pair index
+// p = q*J + j, whatever the scheduling: the sort is deterministic.  No kernel
+// waits for another CTA.  The first pass reads the forward's pair buckets and
+// id rows and drops the pairs of bad ids; its colscan writes the number of
+// valid pairs to stats[0], which the later passes and the reduce read.
+constexpr int kRThreads = 256;
+constexpr int kRWarps = kRThreads / 32;
+constexpr int kRPer = 32;                        // entries per thread and tile
+constexpr int kRWarpKeys = 32 * kRPer;           // entries per warp and tile
+constexpr int kRTile = kRThreads * kRPer;        // entries per tile
+constexpr int kRMaxDigits = 1 << kRadixMaxBits;
+constexpr int kRMaxOwn = kRMaxDigits / kRThreads; // digits per thread at most
+static_assert(kRWarpKeys < 65536, "per-warp digit counts are 16-bit");
+
+// Exclusive scan of one value per thread over a CTA of kRThreads threads.
+__device__ __forceinline__ uint32_t rblock_exclusive_scan(uint32_t v, uint32_t* s_w,
+                                                          uint32_t* total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) s_w[warp] = x;
+    __syncthreads();
+    uint32_t pre = 0, tot = 0;
+#pragma unroll
+    for (int w = 0; w < kRWarps; ++w) {
+        const uint32_t c = s_w[w];
+        pre += (w < warp) ? c : 0u;
+        tot += c;
+    }
+    __syncthreads();
+    *total = tot;
+    return pre + x - v;
+}
+
+// Entry of pair p from its bucket x (kBad for a bad id) and its id's output
+// row: x << 32 | row*J + j, or ~0 when invalid.  Buckets are below 2^32 - 1,
+// so an all-ones entry is never valid.
+template <bool SG>
+__device__ __forceinline__ unsigned long long radix_pair_entry(uint32_t x, uint32_t row,
+                                                               uint32_t p, int J, int log2J) {
+    if (x == kBad) return ~0ull;
+    const uint32_t q = (log2J >= 0) ? (p >> log2J) : p / (uint32_t)J;
+    uint32_t r = row * (uint32_t)J + (p - q * (uint32_t)J);
+    if (SG) {
+        // signed hashing: the sign moves to bit 31 of the entry's low word
+        r |= x & 0x80000000u;
+        x &= 0x7fffffffu;
+    }
+    return ((unsigned long long)x << 32) | r;
+}
+
+template <bool FIRST>
+__device__ __forceinline__ int64_t radix_count(int64_t npairs,
+                                               const unsigned long long* __restrict__ stats) {
+    if (FIRST) return npairs;
+    const unsigned long long v = stats[0];
+    return (int64_t)(v < (unsigned long long)npairs ? v : (unsigned long long)npairs);
+}
+
+// up: cnt[d][tile] = entries of the tile with digit d (every tile writes all
+// of its nd counts, zeros included).
+template <bool FIRST, bool SG>
+__global__ void __launch_bounds__(kRThreads)
+k_radix_up(const uint32_t* __restrict__ pair_x, const unsigned long long* __restrict__ in_e,
+           int64_t npairs, const unsigned long long* __restrict__ stats, int shift, int bits,
+           int ntiles, uint32_t* __restrict__ cnt) {
+    pdl_prologue();
+    __shared__ uint32_t s_c[kRMaxDigits];
+    const int nd = 1 << bits;
+    const uint32_t dmask = (uint32_t)nd - 1u;
+    for (int d = threadIdx.x; d < nd; d += kRThreads) s_c[d] = 0u;
+    __syncthreads();
+    const int64_t n = radix_count<FIRST>(npairs, stats);
+    const int64_t t0 = (int64_t)blockIdx.x * kRTile;
+    uint32_t hi[kRPer];
+#pragma unroll
+    for (int i = 0; i < kRPer; ++i) {
+        const int64_t p = t0 + (int64_t)i * kRThreads + threadIdx.x;
+        if (FIRST) {
+            hi[i] = (p < n) ? __ldg(pair_x + p) : kBad;
+            if (SG && hi[i] != kBad) hi[i] &= 0x7fffffffu;
+        } else {
+            hi[i] = (p < n) ? reinterpret_cast<const uint32_t*>(in_e)[2 * p + 1] : kBad;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < kRPer; ++i)
+        if (hi[i] != kBad) atomicAdd(&s_c[(hi[i] >> shift) & dmask], 1u);
+    __syncthreads();
+    for (int d = threadIdx.x; d < nd; d += kRThreads) cnt[(size_t)d * ntiles + blockIdx.x] = s_c[d];
+}
+
+// colscan: one warp per digit d rewrites the row cnt[d][0 .. ntiles) as its
+// exclusive prefix (the digit's entries in earlier tiles), 512 tiles per round
+// with all of a round's loads in flight; tot[d] = the row's total.  The last
+// CTA to finish writes dstart[d] = sum of tot[d'] over d' < d and returns the
+// ticket counter to zero; with FIRST it also records the number of valid
+// pairs (stats[0]) and clears the distinct-bucket count (stats[1]).
+constexpr int kCsPer = 16;   // tiles per lane and round
+template <bool FIRST>
+__global__ void __launch_bounds__(kRThreads)
+k_radix_colscan(uint32_t* __restrict__ cnt, int ntiles, int bits, uint32_t* __restrict__ tot,
+                uint32_t* __restrict__ dstart, uint32_t* __restrict__ done,
+                unsigned long long* __restrict__ stats) {
+    pdl_prologue();
+    __shared__ uint32_t s_warp[33];
+    __shared__ bool s_last;
+    const int nd = 1 << bits;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int d = blockIdx.x * kRWarps + warp;
+    if (d < nd) {
+        uint32_t* row = cnt + (size_t)d * ntiles;
+        uint32_t carry = 0;
+        for (int t0 = 0; t0 < ntiles; t0 += 32 * kCsPer) {
+            // lane l takes tiles t0 + l*kCsPer .. + kCsPer - 1 (consecutive)
+            uint32_t v[kCsPer];
+            const int tb = t0 + lane * kCsPer;
+#pragma unroll
+            for (int i = 0; i < kCsPer; ++i) v[i] = (tb + i < ntiles) ? row[tb + i] : 0u;
+            uint32_t mine = 0;
+#pragma unroll
+            for (int i = 0; i < kCsPer; ++i) mine += v[i];
+            uint32_t x = mine;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+                if (lane >= o) x += y;
+            }
+            uint32_t run = carry + x - mine;
+#pragma unroll
+            for (int i = 0; i < kCsPer; ++i) {
+                if (tb + i < ntiles) row[tb + i] = run;
+                run += v[i];
+            }
+            carry += __shfl_sync(0xffffffffu, x, 31);
+        }
+        if (lane == 0) tot[d] = carry;
+    }
+    // the last CTA scans the digit totals
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    // nd <= 2048 digits: 8 per thread
+    constexpr int kPer = kRMaxDigits / kRThreads;
+    uint32_t v[kPer], mine = 0;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int dd = threadIdx.x * kPer + i;
+        v[i] = (dd < nd) ? __ldcg(tot + dd) : 0u;
+        mine += v[i];
+    }
+    uint32_t total;
+    uint32_t run = rblock_exclusive_scan(mine, s_warp, &total);
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+        const int dd = threadIdx.x * kPer + i;
+        if (dd < nd) dstart[dd] = run;
+        run += v[i];
+    }
+    if (threadIdx.x == 0) {
+        *done = 0u;
+        if (FIRST) {
+            stats[0] = total;
+            stats[1] = 0;
+        }
+    }
+}
+
+// Shared memory of the down kernel with 2^bits digits.
+__host__ __device__ constexpr size_t radix_down_smem(int nd) {
+    return sizeof(unsigned long long) * kRTile + (sizeof(uint16_t) * kRWarps + 8) * (size_t)nd;
+}
+
+// down: one tile per CTA (see the section comment).
+template <bool FIRST, bool SG>
+__global__ void __launch_bounds__(kRThreads, 2)
+k_radix_down(const uint32_t* __restrict__ pair_x, const uint32_t* __restrict__ q_row,
+             const unsigned long long* __restrict__ in_e, unsigned long long* __restrict__ out_e,
+             int64_t npairs, const unsigned long long* __restrict__ stats, int J, int log2J,
+             int shift, int bits, int ntiles, const uint32_t* __restrict__ cnt,
+             const uint32_t* __restrict__ dstart) {
+    pdl_prologue();
+    extern __shared__ __align__(16) unsigned char r_smem[];
+    const int nd = 1 << bits;
+    unsigned long long* s_tile = reinterpret_cast<unsigned long long*>(r_smem);   // [kRTile]
+    uint16_t* s_hist = reinterpret_cast<uint16_t*>(s_tile + kRTile);               // [kRWarps][nd]
+    uint32_t* s_lst = reinterpret_cast<uint32_t*>(s_hist + kRWarps * nd);          // [nd]
+    uint32_t* s_base = s_lst + nd;                                                 // [nd]
+    __shared__ uint32_t s_w[kRWarps];
+    const uint32_t dmask = (uint32_t)nd - 1u;
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int64_t n = radix_count<FIRST>(npairs, stats);
+    const int64_t t0 = (int64_t)blockIdx.x * kRTile;
+    if (t0 >= n) return;
+    {
+        uint32_t* z = reinterpret_cast<uint32_t*>(s_hist);
+        for (int i = threadIdx.x; i < kRWarps * nd / 2; i += kRThreads) z[i] = 0u;
+    }
+    // load, warp w taking entries t0 + w*kRWarpKeys + i*32 + lane (i in order)
+    unsigned long long e[kRPer];
+    {
+        const int64_t wb = t0 + (int64_t)warp * kRWarpKeys + lane;
+        if (FIRST) {
+            // every load is issued before any is used: buckets, then id rows
+            uint32_t x[kRPer], row[kRPer];
+#pragma unroll
+            for (int i = 0; i < kRPer; ++i) {
+                const int64_t p = wb + i * 32;
+                x[i] = (p < n) ? __ldg(pair_x + p) : kBad;
+            }
+#pragma unroll
+            for (int i = 0; i < kRPer; ++i) {
+                const uint32_t pp = (uint32_t)(wb + i * 32);   // npairs < 2^32 here
+                const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
+                row[i] = (wb + i * 32 < n) ? __ldg(q_row + q) : 0u;
+            }
+#pragma unroll
+            for (int i = 0; i < kRPer; ++i)
+                e[i] = radix_pair_entry<SG>(x[i], row[i], (uint32_t)(wb + i * 32), J, log2J);
+        } else {
+#pragma unroll
+            for (int i = 0; i < kRPer; ++i) {
+                const int64_t p = wb + i * 32;
+                e[i] = (p < n) ? __ldcs(in_e + p) : ~0ull;
+            }
+        }
+    }
+    __syncthreads();
+    // rank each entry among the warp's entries of its digit, in input order
+    uint32_t rank[kRPer];
+    {
+        uint16_t* hw = s_hist + warp * nd;
+        const uint32_t lt = (1u << lane) - 1u;
+#pragma unroll
+        for (int i = 0; i < kRPer; ++i) {
+            const bool valid = e[i] != ~0ull;
+            const uint32_t dg = valid ? ((uint32_t)(e[i] >> (32 + shift)) & dmask) : 0xffffffffu;
+            const uint32_t peers = __match_any_sync(0xffffffffu, dg);
+            const int leader = __ffs(peers) - 1;
+            uint32_t base = 0;
+            if (valid && lane == leader) {
+                base = hw[dg];
+                hw[dg] = (uint16_t)(base + __popc(peers));
+            }
+            base = __shfl_sync(0xffffffffu, base, leader);
+            rank[i] = base + __popc(peers & lt);
+            __syncwarp();
+        }
+    }
+    __syncthreads();
+    // thread t owns digits [t*own, t*own + own) (own = 1 below 256 digits):
+    // warp prefixes, the tile's count of each digit, the digits' starts inside
+    // the tile, and their bases in the output
+    const int own = nd >= kRThreads ? nd / kRThreads : 1;
+    const int d0 = threadIdx.x * own;
+    const bool owner = d0 < nd;
+    uint32_t mine = 0;
+    uint32_t cnt_own[kRMaxOwn];
+#pragma unroll
+    for (int k = 0; k < kRMaxOwn; ++k) {
+        cnt_own[k] = 0;
+        if (k < own && owner) {
+            const int d = d0 + k;
+            uint32_t run = 0;
+#pragma unroll
+            for (int w = 0; w < kRWarps; ++w) {
+                const uint32_t c = s_hist[w * nd + d];
+                s_hist[w * nd + d] = (uint16_t)run;
+                run += c;
+            }
+            cnt_own[k] = run;
+            mine += run;
+        }
+    }
+    uint32_t tile_n;
+    uint32_t lst = rblock_exclusive_scan(mine, s_w, &tile_n);
+#pragma unroll
+    for (int k = 0; k < kRMaxOwn; ++k)
+        if (k < own && owner) {
+            const int d = d0 + k;
+            s_lst[d] = lst;
+            s_base[d] = __ldg(dstart + d) + __ldg(cnt + (size_t)d * ntiles + blockIdx.x) - lst;
+            lst += cnt_own[k];
+        }
+    __syncthreads();
+    // stage the tile in digit order
+#pragma unroll
+    for (int i = 0; i < kRPer; ++i) {
+        if (e[i] == ~0ull) continue;
+        const uint32_t dg = (uint32_t)(e[i] >> (32 + shift)) & dmask;
+        s_tile[s_lst[dg] + s_hist[warp * nd + dg] + rank[i]] = e[i];
+    }
+    __syncthreads();
+    // stores in tile order: the entries of one digit are consecutive in both
+    for (int l = threadIdx.x; l < (int)tile_n; l += kRThreads) {
+        const unsigned long long v = s_tile[l];
+        const uint32_t pos = s_base[(uint32_t)(v >> (32 + shift)) & dmask] + (uint32_t)l;
+        if ((int64_t)pos < npairs) out_e[pos] = v;   // always, when the counts are consistent
     }
 }
 
@@ -385,9 +706,9 @@ constexpr int64_t kPiece = 64;    // sorted entries per reduce task
 template <int VW, int KC, bool JPOW2, bool ZDIV>
 __global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
 k_range_reduce(const unsigned long long* __restrict__ sorted_e,
-               const unsigned long long* __restrict__ stats, int64_t npairs,
+               unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
-               uint32_t smask, bool mixed, double* __restrict__ g, int log2gs) {
+               uint32_t smask, double* __restrict__ g, int log2gs) {
     pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
@@ -426,6 +747,7 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
         __syncwarp(gmask);
     };
 
+    uint32_t nstart = 0;   // distinct buckets: entries whose bucket differs from the one before
     for (int64_t t = (int64_t)blockIdx.x * kWarps * gpw + grp; t < ntasks; t += gstride) {
         const int64_t e0 = t * kPiece;
         const int64_t e1 = (e0 + kPiece < total) ? e0 + kPiece : total;
@@ -439,6 +761,7 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
         for (int u = 0; u < kRU; ++u) nxt[u] = (e0 + u < e1) ? __ldg(sorted_e + e0 + u) : kNone;
         uint32_t cur = (uint32_t)(nxt[0] >> 32);
+        nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
         for (int64_t e = e0; e < e1; e += kRU) {
             uint32_t xs[kRU];
             VT v[kRU][KC];
@@ -486,10 +809,8 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                 }
             }
             // the whole block continues the current run when its last entry
-            // does (entries in bucket order), or, when runs of buckets that
-            // share a counting key may alternate, when every entry does
-            if (xs[kRU - 1] == cur &&
-                (!mixed || (xs[0] == cur && xs[1] == cur && xs[2] == cur))) {
+            // does (entries in bucket order)
+            if (xs[kRU - 1] == cur) {
                 // a tree sum, then one compensated add
 #pragma unroll
                 for (int k = 0; k < KC; ++k)
@@ -506,6 +827,7 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     if (xs[u] != cur) {
                         flush(cur);
                         cur = xs[u];
+                        ++nstart;
                     }
 #pragma unroll
                     for (int k = 0; k < KC; ++k)
@@ -517,6 +839,7 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
         }
         flush(cur);
     }
+    if (lg == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
 }
 
 // Reduce for blocks of at least 32 elements: one WARP per task of kPiece
@@ -532,9 +855,9 @@ static_assert(kWU == 8, "the warp reduce sums kWU = 8 entries as a tree");
 template <int KE, bool ZDIV, bool JPOW2>
 __global__ void __launch_bounds__(kThreads)
 k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
-                    const unsigned long long* __restrict__ stats, int64_t npairs,
+                    unsigned long long* __restrict__ stats, int64_t npairs,
                     const float* __restrict__ gout, int d, int Z, int J, int log2J, int L,
-                    int64_t G, uint32_t smask, bool mixed, double* __restrict__ g) {
+                    int64_t G, uint32_t smask, double* __restrict__ g) {
     pdl_prologue();
     __shared__ unsigned long long s_ent[kWarps][kPiece];
     const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
@@ -554,6 +877,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
             s[k] = c[k] = 0.f;
         }
     };
+    uint32_t nstart = 0;   // distinct buckets: entries whose bucket differs from the one before
     for (int64_t t = (int64_t)blockIdx.x * kWarps + warp; t < ntasks; t += wstride) {
         const int64_t e0 = t * kPiece;
         const int n = (int)((e0 + kPiece < total) ? kPiece : total - e0);
@@ -564,6 +888,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
         for (int k = 0; k < KE; ++k) s[k] = c[k] = 0.f;
         uint32_t cur = (uint32_t)(ent[0] >> 32);
+        nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
         for (int b = 0; b < n; b += kWU) {
             uint32_t xs[kWU];
             float v[kWU][KE];
@@ -590,12 +915,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     v[u][k] = (xs[u] != kBad && z < Lj) ? sign_by(__ldcs(src + z), sb) : 0.f;
                 }
             }
-            bool cont = xs[kWU - 1] == cur;
-            if (mixed) {
-#pragma unroll
-                for (int u = 0; u < kWU - 1; ++u) cont = cont && xs[u] == cur;
-            }
-            if (cont) {
+            if (xs[kWU - 1] == cur) {
 #pragma unroll
                 for (int k = 0; k < KE; ++k) {
                     const float a = (v[0][k] + v[1][k]) + (v[2][k] + v[3][k]);
@@ -609,6 +929,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     if (xs[u] != cur) {
                         flush(cur);
                         cur = xs[u];
+                        ++nstart;
                     }
 #pragma unroll
                     for (int k = 0; k < KE; ++k) kahan_add(s[k], c[k], v[u][k]);
@@ -618,6 +939,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
         flush(cur);
         __syncwarp();
     }
+    if (lane == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
 }
 
 // Reduce for 32-element chunks that tile the rows (Z = 32 dividing d): the
@@ -649,8 +971,8 @@ __device__ __forceinline__ void cp_async_wait() {
 
 __global__ void __launch_bounds__(kThreads)
 k_async_reduce(const unsigned long long* __restrict__ sorted_e,
-               const unsigned long long* __restrict__ stats, int64_t npairs,
-               const float* __restrict__ gout, int64_t G, uint32_t smask, bool mixed,
+               unsigned long long* __restrict__ stats, int64_t npairs,
+               const float* __restrict__ gout, int64_t G, uint32_t smask,
                double* __restrict__ g) {
     pdl_prologue();
     __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
@@ -667,6 +989,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         if (sum != 0.f) red_add_f64(g + (int64_t)x * G + lane, widen(sum));
         sum = comp = 0.f;
     };
+    uint32_t nstart = 0;   // distinct buckets: entries whose bucket differs from the one before
     for (int64_t t = (int64_t)blockIdx.x * kWarps + warp; t < ntasks; t += wstride) {
         const int64_t e0 = t * kAPiece;
         const int n = (int)((e0 + kAPiece < total) ? kAPiece : total - e0);
@@ -698,6 +1021,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         for (int st = 0; st < kAD - 1; ++st) issue(st);
         sum = comp = 0.f;
         uint32_t cur = (uint32_t)(ent[0] >> 32);
+        nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
         for (int st = 0; st < nst; ++st) {
             issue(st + kAD - 1);
             cp_async_wait<kAD - 1>();
@@ -718,12 +1042,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
                 for (int i = 0; i < kAS; ++i) v[i] = sign_by(v[i], ex[2 * i - 1] & smask);
             }
-            // with alternating runs (buckets sharing a counting key) every
-            // entry of the stage is compared, one per lane
-            const bool cont =
-                xlast == cur &&
-                (!mixed || __all_sync(0xffffffffu, ex[2 * (lane & (kAS - 1))] == cur));
-            if (cont) {
+            if (xlast == cur) {
                 const float a = (v[0] + v[1]) + (v[2] + v[3]);
                 const float b = (v[4] + v[5]) + (v[6] + v[7]);
                 kahan_add(sum, comp, a + b);
@@ -737,6 +1056,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                     if (xs[i] != cur) {
                         flush(cur);
                         cur = xs[i];
+                        ++nstart;
                     }
                     kahan_add(sum, comp, v[i]);
                 }
@@ -747,6 +1067,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         cp_async_wait<0>();
         __syncwarp();
     }
+    if (lane == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
 }
 
 template <int KE, bool ZDIV, bool JPOW2>
@@ -757,8 +1078,7 @@ cudaError_t warp_reduce_launch(const SortedBuffers& sb, int64_t npairs, const fl
     const int grid = grid_for(k_warp_range_reduce<KE, ZDIV, JPOW2>, sm_count,
                               (ntasks + kWarps - 1) / kWarps);
     return launch_k(k_warp_range_reduce<KE, ZDIV, JPOW2>, dim3(grid), dim3(kThreads), 0, st,
-                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask,
-                    sb.kmask != 0xffffffffu, g);
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g);
 }
 
 template <int KE>
@@ -782,8 +1102,7 @@ cudaError_t reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* 
     const int64_t work_blocks = (ntasks + gpc - 1) / gpc;
     const int grid = grid_for(k_range_reduce<VW, KC, JPOW2, ZDIV>, sm_count, work_blocks, smem);
     return launch_k(k_range_reduce<VW, KC, JPOW2, ZDIV>, dim3(grid), dim3(kThreads), smem, st,
-                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask,
-                    sb.kmask != 0xffffffffu, g, log2gs);
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g, log2gs);
 }
 
 template <int VW, int KC>
@@ -801,21 +1120,80 @@ cudaError_t reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* go
 
 }  // namespace
 
+RadixPlan radix_plan(uint64_t R, int digit_bits) {
+    // buckets lie in [0, R - 1]: nbits bits with 2^nbits >= R
+    int nbits = 1;
+    while (nbits < 32 && (uint64_t(1) << nbits) < R) ++nbits;
+    const int dmax = digit_bits > 0 ? digit_bits : kRadixMaxBits;
+    RadixPlan pl{};
+    pl.passes = (nbits + dmax - 1) / dmax;
+    const int D = digit_bits > 0 ? digit_bits : (nbits + pl.passes - 1) / pl.passes;
+    for (int k = 0; k < pl.passes; ++k) {
+        pl.shift[k] = k * D;
+        pl.bits[k] = (nbits - k * D) < D ? (nbits - k * D) : D;
+    }
+    return pl;
+}
+
+int64_t radix_tiles(int64_t npairs) {
+    const int64_t t = (npairs + kRTile - 1) / kRTile;
+    return t < 1 ? 1 : t;
+}
+
+template <bool FIRST, bool SG>
+cudaError_t radix_pass(const SortedBuffers& sb, const unsigned long long* in,
+                       unsigned long long* out, int64_t npairs, int J, int log2J,
+                       const RadixPlan& plan, int k, cudaStream_t st) {
+    const int ntiles = (int)radix_tiles(npairs);
+    const int bits = plan.bits[k], shift = plan.shift[k];
+    const int nd = 1 << bits;
+    cudaError_t e = launch_k(k_radix_up<FIRST, SG>, dim3(ntiles), dim3(kRThreads), 0, st,
+                             sb.pair_x, in, npairs, sb.stats, shift, bits, ntiles, sb.cnt);
+    if (e != cudaSuccess) return e;
+    e = launch_k(k_radix_colscan<FIRST>, dim3((nd + kRWarps - 1) / kRWarps), dim3(kRThreads), 0,
+                 st, sb.cnt, ntiles, bits, sb.tot, sb.dstart, sb.done, sb.stats);
+    if (e != cudaSuccess) return e;
+    const size_t smem = radix_down_smem(nd);
+    e = cudaFuncSetAttribute(k_radix_down<FIRST, SG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+    if (e != cudaSuccess) return e;
+    return launch_k(k_radix_down<FIRST, SG>, dim3(ntiles), dim3(kRThreads), smem, st, sb.pair_x,
+                    sb.q_row, in, out, npairs, sb.stats, J, log2J, shift, bits, ntiles, sb.cnt,
+                    sb.dstart);
+}
+
+cudaError_t launch_radix_sort(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
+                              const RadixPlan& plan, cudaStream_t st) {
+    const int log2J = (J & (J - 1)) == 0 ? ceil_log2(J) : -1;
+    const unsigned long long* in = nullptr;
+    for (int k = 0; k < plan.passes; ++k) {
+        // the last pass writes sorted_e; earlier ones alternate with tmp_e
+        unsigned long long* out = ((plan.passes - 1 - k) % 2 == 0) ? sb.sorted_e : sb.tmp_e;
+        cudaError_t e;
+        if (k == 0)
+            e = smask ? radix_pass<true, true>(sb, in, out, npairs, J, log2J, plan, k, st)
+                      : radix_pass<true, false>(sb, in, out, npairs, J, log2J, plan, k, st);
+        else
+            e = radix_pass<false, false>(sb, in, out, npairs, J, log2J, plan, k, st);
+        if (e != cudaSuccess) return e;
+        in = out;
+    }
+    return cudaSuccess;
+}
+
 int64_t sorted_scan_blocks(int64_t R) { return (R + kScanChunk - 1) / kScanChunk; }
-
-
 
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
                                cudaStream_t st) {
     const int64_t nblk = sorted_scan_blocks(R);
     const Touched tc = touched ? *touched : Touched{};
     cudaError_t e = launch_k(k_scan_reduce, dim3((unsigned)nblk), dim3(kScanThreads), 0, st,
-                             sb.cnt, R, sb.bsum, sb.bnz);
+                             sb.ccnt, R, sb.bsum, sb.bnz);
     if (e != cudaSuccess) return e;
     e = launch_k(k_scan_top, dim3(1), dim3(kScanThreads), 0, st, sb.bsum, sb.bnz, nblk, sb.stats,
                  tc.count);
     if (e != cudaSuccess) return e;
-    return launch_k(k_scan_apply, dim3((unsigned)nblk), dim3(kScanThreads), 0, st, sb.cnt, R,
+    return launch_k(k_scan_apply, dim3((unsigned)nblk), dim3(kScanThreads), 0, st, sb.ccnt, R,
                     sb.bsum, sb.bnz, sb.start, tc);
 }
 
@@ -826,11 +1204,11 @@ cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J
     if (smask) {
         const int grid = grid_for(k_sort_scatter<true>, sm_count, nseg);
         return launch_k(k_sort_scatter<true>, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x,
-                        npairs, sb.q_row, J, log2J, sb.kmask, sb.start, sb.cnt, sb.sorted_e);
+                        npairs, sb.q_row, J, log2J, sb.start, sb.ccnt, sb.sorted_e);
     }
     const int grid = grid_for(k_sort_scatter<false>, sm_count, nseg);
     return launch_k(k_sort_scatter<false>, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs,
-                    sb.q_row, J, log2J, sb.kmask, sb.start, sb.cnt, sb.sorted_e);
+                    sb.q_row, J, log2J, sb.start, sb.ccnt, sb.sorted_e);
 }
 
 cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
@@ -838,7 +1216,7 @@ cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_
     const int64_t nseg = (npairs + kSeg - 1) / kSeg;
     const int grid = grid_for(k_sort_count, sm_count, nseg);
     return launch_k(k_sort_count, dim3(grid), dim3(kSegThreads), 0, st, sb.pair_x, npairs, smask,
-                    sb.kmask, sb.cnt);
+                    sb.ccnt);
 }
 
 cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
@@ -856,7 +1234,7 @@ cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const 
         const int64_t ntasks = (npairs + kAPiece - 1) / kAPiece;   // upper bound
         const int grid = grid_for(k_async_reduce, sm_count, (ntasks + kWarps - 1) / kWarps);
         return launch_k(k_async_reduce, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e, sb.stats,
-                        npairs, gout, p.G, p.smask, sb.kmask != 0xffffffffu, g);
+                        npairs, gout, p.G, p.smask, g);
     }
     // blocks of 32+ elements: one warp per task, one element per lane
     if (p.L >= 32) {

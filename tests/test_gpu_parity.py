@@ -420,8 +420,8 @@ def test_compression_sweep(logM, path):
     """Criteo-TB shape with M from 2^18 to 2^33 fp32 (1 MB .. 32 GB).  Up to
     2^26 everything is compared; above, sampled rows and sampled elements
     (touched and untouched) are compared with the oracle evaluated one by one.
-    AUTO takes the sorted path here (above 2^22 block starts its counters are
-    shared by residue); the atomic path is forced at the large sizes too."""
+    AUTO takes the sorted path here (a radix sort of up to three passes); the
+    atomic path is forced at the large sizes too."""
     t = gu.torch()
     M = 1 << logM
     w = wl.make_workload("sweep", M=M)
@@ -481,10 +481,9 @@ def test_compression_sweep(logM, path):
 
 
 # --------------------------------------------------------------------------
-# sorted path with counters shared by residue (more block starts than
-# counters): a small counter count puts hundreds of buckets on each counter,
-# so runs of different buckets alternate inside every residue group
-RESIDUE_CASES = [
+# the deterministic sorted path (stable radix sort), with automatic digits and
+# with narrow ones: 4 or 7 bits per pass give two to six passes
+DIGIT_CASES = [
     dict(name="tb", B=2048),                                  # 32-float chunks, staged reduce
     dict(name="multihot", B=256),                             # multi-id bags
     dict(name="multihot", B=301, bag=("uniform", 0, 6)),      # empty bags, ragged tail
@@ -494,10 +493,10 @@ RESIDUE_CASES = [
 ]
 
 
-@pytest.mark.parametrize("keys", [4, 10])
+@pytest.mark.parametrize("bits", [0, 4, 7])
 @pytest.mark.parametrize("signed", [False, True], ids=["unsigned", "signed"])
-@pytest.mark.parametrize("case", RESIDUE_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
-def test_sorted_residue_keys_parity(case, signed, keys):
+@pytest.mark.parametrize("case", DIGIT_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
+def test_sorted_digit_bits_parity(case, signed, bits):
     from oracle import OraclePSS
     w = _wl(case)
     h, o_u = gu.make_pair(w)
@@ -506,40 +505,43 @@ def test_sorted_residue_keys_parity(case, signed, keys):
         o = OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, signed=True)
         h.set_option(binding.OPT_SIGNED, 1)
     h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
-    h.set_option(binding.OPT_SORT_KEYS, keys)
-    assert h.get_option(binding.OPT_SORT_KEYS) == keys
-    assert h.info()["R"] > (1 << keys)
+    h.set_option(binding.OPT_DETERMINISTIC, 1)
+    h.set_option(binding.OPT_SORT_DIGIT_BITS, bits)
+    assert h.get_option(binding.OPT_SORT_DIGIT_BITS) == bits
+    assert h.info()["R"] > (1 << bits)             # at least two passes when narrow
     idx, off = _batch_cuda(w)
     out = gu.host(h.forward(idx, off, w.B)).ravel()
     ref, _ = o.forward(w.w0, w.indices, w.offsets, w.B)
-    gu.check_forward(out, ref, _abs_pool(o_u, w.w0, w), what="residue forward")
+    gu.check_forward(out, ref, _abs_pool(o_u, w.w0, w), what="narrow-digit forward")
     g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
     A = o_u.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
-    gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, w.grad_out), A, what="residue grad")
+    gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, w.grad_out), A, what="narrow-digit grad")
     assert h.info()["last_path"] == binding.PATH_SORTED
-    # a step with each update pass: the touched one lists the buckets from the pairs
+    # a step with each update pass
     for mode in (binding.UPDATE_TOUCHED, binding.UPDATE_DENSE):
         h.set_state(gu.cuda(w.w0), gu.cuda(np.zeros(w.M, np.float32)) if w.opt == "adagrad" else None)
         h.set_option(binding.OPT_UPDATE_MODE, mode)
         wg, Gg, w2, G2, g32, _ = _run_step(w, h, o, w.w0, np.zeros(w.M, np.float32),
                                            (w.indices, w.offsets, w.grad_out))
         if w.opt == "sgd":
-            gu.check_sgd(wg, w2, A, w.lr, what=f"residue sgd, update mode {mode}")
+            gu.check_sgd(wg, w2, A, w.lr, what=f"narrow-digit sgd, update mode {mode}")
         else:
-            gu.check_adagrad(wg, Gg, w2, G2, g32, A, w.lr, what=f"residue adagrad, update mode {mode}")
+            gu.check_adagrad(wg, Gg, w2, G2, g32, A, w.lr,
+                             what=f"narrow-digit adagrad, update mode {mode}")
     assert h.get_error() == (binding.PSS_OK, -1)
     h.close()
 
 
 @pytest.mark.parametrize("opt", ["sgd", "adagrad"])
-def test_sorted_residue_keys_dyadic_bit_exact(opt):
-    # dyadic inputs: every sum is exact, so alternating runs must still give
+def test_sorted_narrow_digits_dyadic_bit_exact(opt):
+    # dyadic inputs: every sum is exact, so a five-pass sort must still give
     # the oracle's bits
     w = wl.make_workload("kaggle", B=1024, grad="dyadic", w0="dyadic")
     w.lr = 0.125
     h, o = gu.make_pair(w, opt=opt)
     h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
-    h.set_option(binding.OPT_SORT_KEYS, 6)
+    h.set_option(binding.OPT_DETERMINISTIC, 1)
+    h.set_option(binding.OPT_SORT_DIGIT_BITS, 4)
     h.forward(*_batch_cuda(w), w.B)
     h.backward_update(gu.cuda(w.grad_out), w.lr)
     wg, Gg = h.get_state()
@@ -551,22 +553,25 @@ def test_sorted_residue_keys_dyadic_bit_exact(opt):
     h.close()
 
 
-def test_sort_keys_option_rules():
+def test_sort_digit_bits_option_rules():
     w = wl.make_workload("tiny")
     h, _ = gu.make_pair(w)
-    assert h.get_option(binding.OPT_SORT_KEYS) == 22
-    for bad in (3, 31, -1):
+    assert h.get_option(binding.OPT_SORT_DIGIT_BITS) == 0
+    assert h.get_option(binding.OPT_DETERMINISTIC) == 0
+    for bad in (2, -1):
+        with pytest.raises(binding.PSSError):
+            h.set_option(binding.OPT_DETERMINISTIC, bad)
+    h.set_option(binding.OPT_DETERMINISTIC, 1)
+    assert h.get_option(binding.OPT_DETERMINISTIC) == 1
+    for bad in (1, 3, 12, -1):
         with pytest.raises(binding.PSSError) as e:
-            h.set_option(binding.OPT_SORT_KEYS, bad)
+            h.set_option(binding.OPT_SORT_DIGIT_BITS, bad)
         assert e.value.status == binding.PSS_ERR_INVALID_ARG
     h.forward(*_batch_cuda(w), w.B)
-    h.set_option(binding.OPT_SORT_KEYS, 22)          # unchanged: the batch stays
+    h.set_option(binding.OPT_SORT_DIGIT_BITS, 4)     # the batch stays: nothing depends on it
     h.backward_update(gu.cuda(w.grad_out), w.lr)
-    h.forward(*_batch_cuda(w), w.B)
-    h.set_option(binding.OPT_SORT_KEYS, 8)           # changed: the batch is forgotten
-    with pytest.raises(binding.PSSError) as e:
-        h.backward_update(gu.cuda(w.grad_out), w.lr)
-    assert e.value.status == binding.PSS_ERR_STATE
+    h.set_option(binding.OPT_SORT_DIGIT_BITS, 11)
+    assert h.get_option(binding.OPT_SORT_DIGIT_BITS) == 11
     h.close()
 
 
@@ -705,16 +710,17 @@ def test_circular_forward_and_grad_parity(case, path, signed):
 @pytest.mark.parametrize("signed", [False, True], ids=["unsigned", "signed"])
 @pytest.mark.parametrize("case", [dict(name="tb", B=2048), dict(name="kaggle", Z=3, G=2, B=300)],
                          ids=["tb", "kaggle-Z3-G2"])
-def test_circular_with_residue_keys(case, signed):
-    # circular array and counters shared by residue (64 counters): the wrapped
-    # blocks' contributions fold into the head after alternating runs
+def test_circular_with_narrow_digits(case, signed):
+    # circular array and a many-pass radix sort: the wrapped blocks'
+    # contributions fold into the head after the sorted reduce
     w = _wl(case)
     h, o, o_abs = _circ_pair(w, "sorted", signed)
-    h.set_option(binding.OPT_SORT_KEYS, 6)
+    h.set_option(binding.OPT_DETERMINISTIC, 1)
+    h.set_option(binding.OPT_SORT_DIGIT_BITS, 5)
     h.forward(*_batch_cuda(w), w.B)
     g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
     A = o_abs.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
-    gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, w.grad_out), A, what="circular residue grad")
+    gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, w.grad_out), A, what="circular narrow-digit grad")
     assert h.info()["last_path"] == binding.PATH_SORTED
     h.close()
 
@@ -925,5 +931,12 @@ def test_profile_and_launch_counts():
     h.backward_update(go, w.lr)
     assert h.profile(binding.K_SORT)[0] == 1 and h.profile(binding.K_REDUCE)[0] == 1
     # forward, bucket count, 3 scan kernels, slot scatter, reduce, update
+    assert h.info()["R"] < (1 << 22)
     assert h.info()["kernel_launches"] - before == 8
+    # deterministic: forward, two radix passes of three kernels each (R < 2^22), reduce, update
+    h.set_option(binding.OPT_DETERMINISTIC, 1)
+    before = h.info()["kernel_launches"]
+    h.forward(idx, off, w.B)
+    h.backward_update(go, w.lr)
+    assert h.info()["kernel_launches"] - before == 9
     h.close()
