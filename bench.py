@@ -50,6 +50,65 @@ WORKLOAD_DESC = {
 }
 
 
+def _host():
+    """Host cores and CPU model (for the CPU-oracle baseline)."""
+    model = None
+    try:
+        with open("/proc/cpuinfo") as f:
+            info = f.read()
+        for key in ("model name", "Hardware", "cpu model"):
+            m = re.search(rf"^{key}\s*:\s*(.+)$", info, flags=re.M)
+            if m:
+                model = m.group(1).strip()
+                break
+        if model is None:
+            impl = re.search(r"^CPU implementer\s*:\s*(\S+)", info, flags=re.M)
+            part = re.search(r"^CPU part\s*:\s*(\S+)", info, flags=re.M)
+            if impl and part:
+                model = f"arm implementer {impl.group(1)} part {part.group(1)}"
+    except OSError:
+        pass
+    if model is None:
+        import platform
+        model = platform.processor() or platform.machine()
+    return {"nproc": os.cpu_count(), "cpu_model": model}
+
+
+def _l2_peaks(torch, dev, sm_count):
+    """L2 rates measured live with the library's probe kernels over a 32 MB
+    device buffer (L2-resident): uniformly random 128-byte block gathers (the
+    L2 peak of the roofline: the forward's block reads have this shape),
+    streaming 128-byte line reads, and fp64 / 16-byte fp32 reductions into
+    random 32-lane blocks (consecutive elements per instruction, as the
+    kernels issue them).  Best of 5 timed calls after 2 warm-up calls, CUDA
+    events on the launch stream."""
+    from paper_2207_10731_gb300 import binding
+    nbytes = 32 << 20
+    buf = torch.zeros(nbytes // 4, dtype=torch.float32, device=dev)
+    ctas = sm_count * 16
+    stream = torch.cuda.current_stream()
+    out = {"buffer_mb": nbytes >> 20, "ctas": ctas}
+    for kind, iters, key in ((0, 1024, "gather_gbs"), (3, 1024, "read_gbs"),
+                             (1, 256, "red_f64_adds_per_s"), (2, 256, "red_v4_f32_adds_per_s")):
+        best = None
+        for rep_ in range(7):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            binding.probe_l2(kind, buf, iters, ctas, stream)
+            b.record(stream)
+            torch.cuda.synchronize()
+            if rep_ >= 2:
+                ms = a.elapsed_time(b)
+                best = ms if best is None else min(best, ms)
+        if kind in (0, 3):
+            it = -(-iters // 8) * 8
+            out[key] = ctas * 8 * it * 128 / (best / 1e3) / 1e9
+        else:
+            out[key] = ctas * 256 * iters * (4 if kind == 2 else 1) / (best / 1e3)
+    del buf
+    return out
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -179,6 +238,22 @@ def _algorithmic_bytes(w: wl.Workload):
     }
 
 
+def _step_roofline(ab, step_s, hbm_peak, l2, forward_only, array_in_l2):
+    """The step's bound: HBM time of its streamed bytes against L2 time of its
+    shared-array gathers and adds (when the array is L2-resident), the larger
+    of the two; frac = that bound over the measured step time."""
+    hbm_bytes = ab["forward"] if forward_only else ab["step"]
+    l2_bytes = ab["l2_gather"] + (0 if forward_only else ab["l2_scatter"])
+    t_hbm = hbm_bytes / (hbm_peak * 1e9)
+    t_l2 = l2_bytes / (l2["gather_gbs"] * 1e9) if (l2 and array_in_l2) else 0.0
+    bound = "l2" if t_l2 > t_hbm else "hbm"
+    return {"bound": bound, "t_hbm_ms": t_hbm * 1e3, "t_l2_ms": t_l2 * 1e3,
+            "hbm_bytes": hbm_bytes, "l2_bytes": l2_bytes if array_in_l2 else None,
+            "frac": max(t_hbm, t_l2) / step_s, "target_frac": 0.60,
+            "note": "fused forward + backward + update against max(HBM time, L2 time); "
+                    "L2 time uses the measured random 128-byte L2 gather rate"}
+
+
 def _oracle_sample(w: wl.Workload, rows: int):
     """First ``rows`` batch rows of every table as a smaller batch."""
     idx_parts, lens = [], []
@@ -301,7 +376,7 @@ def run_reference(args):
         "config": dict({"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B, "seq_len": 1,
                         "parallelism": "single host thread"}, **_config_extra(args, w)),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": sample},
+                         "host": _host(), "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -440,6 +515,12 @@ def run_gpu(args):
     h2d = int(np.mean([i.nbytes + o.nbytes + (0 if args.forward_only else g.nbytes)
                        for i, o, g in batches]))
     d2h = int(hout.numel() * 4)
+    props = torch.cuda.get_device_properties(dev)
+    l2 = _l2_peaks(torch, dev, props.multi_processor_count) if rank == 0 else None
+    # the shared array's working set (w, the Adagrad accumulator and the fp64
+    # gradient: 16 bytes per element) fits in L2
+    l2_size = getattr(props, "L2_cache_size", 0) or (126 << 20)
+    array_in_l2 = 16 * w.M <= l2_size // 2
 
     if rank == 0:
         clocks = sampler.summary(wall0, wall2) if sampler else None
@@ -454,13 +535,27 @@ def run_gpu(args):
         avg_s = ms_dom / max(1, n_dom) / 1e3
         bytes_dom = ab[dom]
         achieved = bytes_dom / avg_s / 1e9
+        kroof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
+                 "unit": "GB/s", "frac": achieved / peak, "traffic": _traffic(dom, args.workload),
+                 "peak_kind": peak_kind, "algorithmic_bytes_per_launch": bytes_dom,
+                 "avg_launch_ms": avg_s * 1e3}
+        if dom == "forward" and array_in_l2 and l2:
+            # the forward's block gathers from the L2-resident array take
+            # longer at the measured L2 gather rate than its HBM streams
+            t_l2 = ab["l2_gather"] / (l2["gather_gbs"] * 1e9)
+            if t_l2 > bytes_dom / (peak * 1e9):
+                a_l2 = ab["l2_gather"] / avg_s / 1e9
+                kroof.update({"bound": "l2", "achieved": a_l2, "peak": l2["gather_gbs"],
+                              "frac": a_l2 / l2["gather_gbs"],
+                              "peak_kind": "measured (L2 random 128-byte gather probe)",
+                              "algorithmic_bytes_per_launch": ab["l2_gather"], "traffic": None})
         step_bytes = ab["forward"] if args.forward_only else ab["step"]
         step_gbs = step_bytes / (elapsed_ms / args.steps / 1e3) / 1e9 * world
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             rate, rows, reps, nnz_s, tot = _oracle_rate(w, args.cpu_budget, args.forward_only,
                                                         signed=args.signed)
-            cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
+            cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle", "host": _host(),
                    "sample": (f"first {rows} of {w.B} batch rows x {w.T} tables "
                               f"({nnz_s} lookups) per step, {reps} steps, {tot:.1f} s: "
                               + ("forward only" if args.forward_only else
@@ -481,12 +576,10 @@ def run_gpu(args):
                        **_config_extra(args, w)},
             "step_gbs": step_gbs,
             "bags_per_s": w.B * w.T * args.steps * world / (elapsed_ms / 1e3),
-            "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
-                         "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": _traffic(dom, args.workload),
-                         "peak_kind": peak_kind, "algorithmic_bytes_per_launch": bytes_dom,
-                         "avg_launch_ms": avg_s * 1e3,
-                         "step_frac": step_gbs / world / peak},
+            "roofline": dict(kroof, step_frac=step_gbs / world / peak),
+            "step_roofline": _step_roofline(ab, elapsed_ms / args.steps / 1e3, peak, l2,
+                                            args.forward_only, array_in_l2),
+            "l2_peaks": l2,
             "kernels_ms": {k: v[1] / v[0] for k, v in prof.items()},
             "kernel_split": {"steps": split_steps, "ms_per_step_with_events": split_ms / split_steps,
                              "note": "kernels_ms and roofline.avg_launch_ms come from a second "

@@ -90,8 +90,9 @@ typedef enum {
      * accumulation bound; dyadic inputs give identical bits).  The sorted path
      * groups the contributions by location and sums each location's run once
      * (see PSS_OPT_DETERMINISTIC for its order).  PSS_PATH_AUTO takes the
-     * sorted path when the batch adds at least 2^23 elements (nnz * J * L),
-     * the atomic one below (crossover measured on GB300; M does not move it). */
+     * sorted path when the batch adds at least 5,000,000 elements (nnz * J *
+     * L) with blocks of L >= 32 elements, 10,000,000 with shorter blocks, the
+     * atomic one below (crossovers measured on GB300; M does not move them). */
     PSS_OPT_BACKWARD_PATH = 1,
     /* How the Adagrad step visits M: every element (PSS_UPDATE_DENSE), only the
      * blocks the batch touched (PSS_UPDATE_TOUCHED), or chosen from M and the
@@ -337,6 +338,31 @@ pss_status pss_grad_noalloc(const int64_t* table_cardinalities, int32_t num_tabl
  */
 pss_status pss_check_convert(int32_t direction, const void* in, void* out, int64_t n,
                              pss_stream stream);
+
+/*
+ * L2 rate probe (the paper has no counterpart: a measurement hook of this
+ * library, used for the L2 roofline).  Queues one kernel of `ctas` CTAs of 256
+ * threads on `stream` over the caller's DEVICE buffer `buf` of `bytes` bytes
+ * (256-byte aligned, at least 4096; its contents are overwritten):
+ *   kind 0: every warp reads `iters` (rounded up to a multiple of 8) random
+ *           128-byte blocks of buf (lane l reads word l of the block), among
+ *           the first power-of-two number of blocks that fits;
+ *   kind 1: every warp adds 1.0 into `iters` random blocks of 32 consecutive
+ *           doubles of buf, one per lane (red.global.add.f64), among the
+ *           first power-of-two number of blocks that fits;
+ *   kind 2: likewise (1,1,1,1) into blocks of 32 consecutive 16-byte fp32
+ *           vectors (red.global.add.v4.f32);
+ *   kind 3: like kind 0, but the warps read consecutive 128-byte lines
+ *           (a streaming read of buf, wrapping around).
+ * The caller times the call with events on `stream`; bytes moved = ctas * 8 *
+ * iters * 128 (kinds 0 and 3), adds = ctas * 256 * iters (kind 1) or 4x that
+ * (kind 2).  Buffers below 512 bytes per block are refused for kinds 1 and 2
+ * only through the 4096-byte minimum.
+ * Errors: PSS_ERR_INVALID_ARG (kind, sizes, alignment, a host buffer),
+ * PSS_ERR_CUDA.
+ */
+pss_status pss_probe_l2(int32_t kind, void* buf, int64_t bytes, int64_t iters, int32_t ctas,
+                        pss_stream stream);
 
 #ifdef __cplusplus
 }

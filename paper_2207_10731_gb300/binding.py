@@ -39,7 +39,7 @@ EXPORTS = [
     "pss_set_state", "pss_compute_locations", "pss_forward", "pss_backward_update",
     "pss_backward_grad", "pss_set_option", "pss_get_option", "pss_get_error", "pss_get_info",
     "pss_get_profile", "pss_reset_profile", "pss_status_string", "pss_grad_noalloc",
-    "pss_check_convert",
+    "pss_check_convert", "pss_probe_l2",
 ]
 
 
@@ -97,6 +97,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "pss_grad_noalloc": [vp, i32, i32, i64, i32, i32, u64, vp, i64, vp, i64, vp, vp, vp,
                                  vp],
             "pss_check_convert": [i32, vp, vp, i64, vp],
+            "pss_probe_l2": [i32, vp, i64, i64, i32, vp],
         }
         for name, args in sigs.items():
             fn = getattr(lib, name)
@@ -106,6 +107,13 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         lib.pss_status_string.restype = ctypes.c_char_p
         _lib = lib
         return lib
+
+
+def probe_l2(kind: int, buf, iters: int, ctas: int, stream=None):
+    """Queue one L2 rate probe kernel (pss_probe_l2) over the device tensor buf."""
+    lib = load_library()
+    _check(lib.pss_probe_l2(int(kind), _ptr(buf), buf.numel() * buf.element_size(), int(iters),
+                            int(ctas), _stream_ptr(stream)), "pss_probe_l2")
 
 
 def status_string(status: int) -> str:

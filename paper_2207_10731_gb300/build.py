@@ -20,7 +20,8 @@ OUT_DIR = os.path.join(PKG, "_lib")
 OBJ_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(OUT_DIR, "libpss.so")
 
-SOURCES = ["pss_api.cu", "pss_kernels.cu", "pss_tiled.cu", "pss_sorted.cu", "pss_noalloc.cu"]
+SOURCES = ["pss_api.cu", "pss_kernels.cu", "pss_tiled.cu", "pss_sorted.cu", "pss_noalloc.cu",
+           "pss_probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -346,14 +346,17 @@ bool use_touched(const pss_handle* h, int64_t pairs) {
 // The sorted path holds bucket indices in 32 bits, 0xffffffff marking a bad
 // id: it needs R < kSortedMaxR, the bound below which the forward emits 32-bit
 // buckets at all.  AUTO takes the sorted path when the batch adds at least
-// kAutoSortedMinAdds elements (pairs * L): measured on GB300, the atomic path
-// wins below it (its one kernel against the sort's launches; Criteo-Kaggle
-// shape at batch 8192: 3.4M adds, 0.049 against 0.108 ms per step), the sorted
-// path above it at every M from 2^18 to 2^33, Zipf or uniform ids
-// (Criteo-Kaggle shape at batch 32768 and Criteo-TB shape at batch 4096: 13.6M
-// adds, 0.138 against 0.186 and 0.073 against 0.113 ms).
+// auto_sorted_min_adds(L) elements (pairs * L), the atomic path below: the
+// atomic path's one kernel wins small batches, the sorted path's sort and
+// reduce win large ones at every M from 2^18 to 2^33, Zipf or uniform ids.
+// Measured on GB300 (ms per step, atomic against sorted):
+//   L = 32, Criteo-TB shape:     3.4M adds 0.045 / 0.055, 6.8M adds 0.074 / 0.059
+//   L = 16, Criteo-Kaggle shape: 6.8M adds 0.087 / 0.118, 13.6M adds 0.186 / 0.138
+// (blocks shorter than a warp leave the sorted reduce's lanes partly idle, so
+// its crossover lies higher).
 constexpr int64_t kSortedMaxR = int64_t(0xffffffffLL);
-constexpr int64_t kAutoSortedMinAdds = int64_t(1) << 23;
+
+int64_t auto_sorted_min_adds(int32_t L) { return L >= 32 ? 5000000 : 10000000; }
 
 bool sorted_supported(const pss_handle* h, int64_t nnz, int64_t B) {
     const int64_t J = h->dp.J;
@@ -373,7 +376,7 @@ bool use_radix(const pss_handle* h) {
 bool want_sorted(const pss_handle* h, int64_t npairs) {
     if (h->path == PSS_PATH_SORTED) return true;
     if (h->path == PSS_PATH_ATOMIC) return false;
-    return npairs * (int64_t)h->dp.L >= kAutoSortedMinAdds;
+    return npairs * (int64_t)h->dp.L >= auto_sorted_min_adds(h->dp.L);
 }
 
 pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {

@@ -957,9 +957,24 @@ constexpr int kAD = 4;          // ring slots (kAD - 1 stages in flight)
 // tasks per warp: that reduce took 77 against 57 us.
 constexpr int kAPiece = 128;
 
-__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+// L2 policy for data read once (the upstream gradient, the sorted entries):
+// evicted first, so that the streams do not push the fp64 accumulator and the
+// shared array out of L2.
+__device__ __forceinline__ uint64_t l2_evict_first() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, uint64_t pol) {
     const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" :: "r"(sa), "l"(gmem) : "memory");
+    asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;\n"
+                 :: "r"(sa), "l"(gmem), "l"(pol) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_once_u64(const unsigned long long* p,
+                                                          uint64_t pol) {
+    unsigned long long v;
+    asm volatile("ld.global.nc.L2::cache_hint.u64 %0, [%1], %2;" : "=l"(v) : "l"(p), "l"(pol));
+    return v;
 }
 __device__ __forceinline__ void cp_async_commit() {
     asm volatile("cp.async.commit_group;\n" ::: "memory");
@@ -984,6 +999,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
     unsigned long long* ent = s_ent[warp];
     const int64_t wstride = (int64_t)gridDim.x * kWarps;
     constexpr unsigned long long kNone = (unsigned long long)kBad << 32;
+    const uint64_t pol = l2_evict_first();
     float sum = 0.f, comp = 0.f;
     auto flush = [&](uint32_t x) {
         if (sum != 0.f) red_add_f64(g + (int64_t)x * G + lane, widen(sum));
@@ -995,7 +1011,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         const int n = (int)((e0 + kAPiece < total) ? kAPiece : total - e0);
 #pragma unroll
         for (int h = 0; h < kAPiece; h += 32)
-            ent[h + lane] = (h + lane < n) ? __ldg(sorted_e + e0 + h + lane) : kNone;
+            ent[h + lane] = (h + lane < n) ? ld_once_u64(sorted_e + e0 + h + lane, pol) : kNone;
         __syncwarp();
         const int nst = (n + kAS - 1) / kAS;
         // copy stage st (kAS chunks of 128 bytes = 64 pieces of 16 bytes)
@@ -1011,7 +1027,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                         const uint32_t r =
                             reinterpret_cast<const uint32_t*>(ent)[2 * e] & ~smask;  // low word
                         cp_async16(&s_ring[warp][st % kAD][i][part * 4],
-                                   gout + (uint64_t)r * 32u + (uint32_t)(part * 4));
+                                   gout + (uint64_t)r * 32u + (uint32_t)(part * 4), pol);
                     }
                 }
             }

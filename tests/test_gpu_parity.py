@@ -940,3 +940,36 @@ def test_profile_and_launch_counts():
     h.backward_update(go, w.lr)
     assert h.info()["kernel_launches"] - before == 9
     h.close()
+
+
+def test_l2_probe_runs_and_rejects_bad_arguments():
+    # the measurement hook behind bench.py's L2 peaks: every kind runs on a
+    # device buffer; host buffers, bad kinds and unaligned sizes are refused
+    t = gu.torch()
+    buf = t.zeros(1 << 20, dtype=t.float32, device="cuda")
+    for kind in (0, 1, 2, 3):
+        binding.probe_l2(kind, buf, 16, 8)
+    t.cuda.synchronize()
+    for bad in (dict(kind=4, buf=buf), dict(kind=0, buf=t.zeros(1 << 20))):
+        with pytest.raises(binding.PSSError) as e:
+            binding.probe_l2(bad["kind"], bad["buf"], 16, 8)
+        assert e.value.status == binding.PSS_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("name,B,want", [("tb", 1024, "atomic"), ("tb", 2048, "sorted"),
+                                          ("kaggle", 8192, "atomic"),
+                                          ("kaggle", 32768, "sorted")])
+def test_auto_path_threshold(name, B, want):
+    # AUTO picks the sorted path from 5M element adds (nnz * J * L) with
+    # 32-element blocks and from 10M with shorter ones: the Criteo-TB shape
+    # adds 3.4M at batch 1024 and 6.8M at 2048, the Criteo-Kaggle shape
+    # (16-element blocks) 3.4M at batch 8192 and 13.6M at 32768
+    w = wl.make_workload(name, B=B)
+    h, o = gu.make_pair(w)
+    assert h.get_option(binding.OPT_BACKWARD_PATH) == binding.PATH_AUTO
+    h.forward(*_batch_cuda(w), w.B)
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    assert h.info()["last_path"] == PATHS[want]
+    gu.check_grad(g, o.grad(w.indices, w.offsets, w.B, w.grad_out),
+                  o.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out)))
+    h.close()
