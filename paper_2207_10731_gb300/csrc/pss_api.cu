@@ -390,7 +390,7 @@ pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {
         h->sb_fixed = true;
     }
     if (h->sb_pairs_cap < npairs) {
-        for (void** b : {(void**)&h->sb.pair_x, (void**)&h->sb.sorted_e}) {
+        for (void** b : {(void**)&h->sb.pair_x, (void**)&h->sb.sorted_e, (void**)&h->sb.bnd}) {
             if (*b) PSS_TRY(cudaFreeAsync(*b, st));
             *b = nullptr;
         }
@@ -398,6 +398,8 @@ pss_status ensure_sorted(pss_handle* h, int64_t nnz, cudaStream_t st) {
         const size_t n = (size_t)(npairs > 0 ? npairs : 1);
         PSS_TRY(cudaMallocAsync(&h->sb.pair_x, sizeof(uint32_t) * n, st));
         PSS_TRY(cudaMallocAsync(&h->sb.sorted_e, sizeof(unsigned long long) * n, st));
+        PSS_TRY(cudaMallocAsync(&h->sb.bnd, sizeof(float) * 64 * (size_t)window_records((int64_t)n),
+                                st));
         h->sb_pairs_cap = npairs;
     }
     if (h->sb_ids_cap < nnz) {
@@ -597,7 +599,7 @@ pss_status pss_destroy(pss_handle* h) {
                     (void*)h->sb.tmp_e, (void*)h->sb.cnt, (void*)h->sb.tot,
                     (void*)h->sb.dstart, (void*)h->sb.done, (void*)h->sb.stats,
                     (void*)h->sb.ccnt, (void*)h->sb.start, (void*)h->sb.bsum,
-                    (void*)h->sb.bnz})
+                    (void*)h->sb.bnz, (void*)h->sb.bnd})
         if (b) cudaFree(b);
     if (h->stats_host) cudaFreeHost(h->stats_host);
     if (h->stats_ev) cudaEventDestroy(h->stats_ev);
@@ -755,11 +757,10 @@ static pss_status scatter_into(pss_handle* h, const float* dgrad, float scale, f
                                       touch ? &h->touched : nullptr, h->err, h->sm_count, st));
 }
 
-// Sorted path: sort by bucket (counting or radix), segmented reduce into g64.
-static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, bool touch,
-                                cudaStream_t st) {
+// Sorted path, step 1: sort the last forward's pairs by bucket (counting or
+// radix sort); with `touch`, also list the touched blocks.
+static pss_status sort_pairs(pss_handle* h, bool touch, cudaStream_t st) {
     const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
-    if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
     poll_stats(h);
     if (use_radix(h)) {
         pss_status rc0 = ensure_radix(h, npairs, st);
@@ -779,6 +780,54 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, 
         PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, touch ? &h->touched : nullptr, st));
         PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->dp.smask, h->sm_count, st));
     }
+    return PSS_OK;
+}
+
+// Valid pairs (the sort) and distinct buckets (the reduce), for
+// pss_get_info's collision rate; one copy in flight at a time.
+static pss_status copy_stats(pss_handle* h, cudaStream_t st) {
+    if (!h->stats_pending) {
+        PSS_TRY(cudaMemcpyAsync(h->stats_host, h->sb.stats, 2 * sizeof(unsigned long long),
+                                cudaMemcpyDeviceToHost, st));
+        PSS_TRY(cudaEventRecord(h->stats_ev, st));
+        h->stats_pending = true;
+    }
+    return PSS_OK;
+}
+
+// Sorted path with the window reduce: sort (with `touch`, also list the
+// touched blocks), then every element's gradient stored once into gexp
+// (fp32, zero on entry).
+static pss_status sorted_window(pss_handle* h, const float* dgrad, bool staged, bool touch,
+                                float* gexp, cudaStream_t st) {
+    const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
+    if (h->dp.T * h->last_B == 0 || npairs == 0) return grad_wait(h, staged, st);
+    pss_status rc = sort_pairs(h, touch, st);
+    if (rc != PSS_OK) return rc;
+    if ((rc = grad_wait(h, staged, st)) != PSS_OK) return rc;
+    {
+        LaunchScope ls(h, PSS_K_REDUCE, st, 2);
+        const WindowSink ws{gexp, h->sb.bnd};
+        PSS_TRY(launch_window_reduce(h->sb, npairs, dgrad, h->dp, ws, h->sm_count, st));
+    }
+    return copy_stats(h, st);
+}
+
+// The fp32 gradient buffer of the window reduce (zero between calls).
+static pss_status ensure_g32(pss_handle* h, cudaStream_t st) {
+    if (h->g) return PSS_OK;
+    PSS_TRY(cudaMalloc(&h->g, sizeof(float) * (size_t)(h->dp.M + h->dp.L)));
+    PSS_TRY(cudaMemsetAsync(h->g, 0, sizeof(float) * (size_t)(h->dp.M + h->dp.L), st));
+    return PSS_OK;
+}
+
+// Sorted path: sort by bucket (counting or radix), segmented reduce into g64.
+static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, bool touch,
+                                cudaStream_t st) {
+    const int64_t npairs = h->last_nnz * (int64_t)h->dp.J;
+    if (h->dp.T * h->last_B == 0 || npairs == 0) return PSS_OK;
+    pss_status rc0 = sort_pairs(h, touch, st);
+    if (rc0 != PSS_OK) return rc0;
     // the sort above needs only the forward's buckets: a host gradient's copy
     // has overlapped it, and is waited for here
     pss_status rc = grad_wait(h, staged, st);
@@ -787,15 +836,7 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, 
         LaunchScope ls(h, PSS_K_REDUCE, st);
         PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64, h->sm_count, st));
     }
-    // valid pairs (the sort) and distinct buckets (the reduce), for
-    // pss_get_info's collision rate; one copy in flight at a time
-    if (!h->stats_pending) {
-        PSS_TRY(cudaMemcpyAsync(h->stats_host, h->sb.stats, 2 * sizeof(unsigned long long),
-                                cudaMemcpyDeviceToHost, st));
-        PSS_TRY(cudaEventRecord(h->stats_ev, st));
-        h->stats_pending = true;
-    }
-    return PSS_OK;
+    return copy_stats(h, st);
 }
 
 pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, pss_stream stream) {
@@ -813,7 +854,28 @@ pss_status pss_backward_update(pss_handle* h, const float* grad_out, float lr, p
     const bool ada = h->opt == PSS_ADAGRAD;
     const bool sorted = h->batch_emitted && want_sorted(h, h->last_nnz * (int64_t)h->dp.J);
     h->last_path = sorted ? PSS_PATH_SORTED : PSS_PATH_ATOMIC;
-    if (sorted) {
+    if (sorted && h->deterministic && !h->circ && window_reduce_ok(h->dp, dg)) {
+        // each element's gradient stored once into the fp32 buffer, then the
+        // update pass (which returns the buffer to zero)
+        if ((rc = ensure_g32(h, st)) != PSS_OK) return rc;
+        const bool touch = use_touched(h, pairs);
+        if (touch && (rc = ensure_touched(h, pairs, st)) != PSS_OK) return rc;
+        if ((rc = sorted_window(h, dg, staged, touch, h->g, st)) != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
+        {
+            LaunchScope ls(h, PSS_K_UPDATE, st);
+            if (touch)
+                PSS_TRY(launch_update_touched(ada, h->w, h->Gacc, h->g, h->touched, h->dp.G,
+                                              h->dp.L, lr, h->eps, h->sm_count, st));
+            else
+                PSS_TRY(launch_update_dense(ada, h->w, h->Gacc, h->g, h->dp.M, lr, h->eps,
+                                            h->sm_count, st));
+        }
+        if (touch) {
+            LaunchScope ls(h, PSS_K_MISC, st);
+            PSS_TRY(launch_touched_clear(h->touched, h->sm_count, st));
+        }
+    } else if (sorted) {
         const int64_t saved = h->accum;
         h->accum = PSS_ACCUM_F64;                 // the sorted path sums into g64
         rc = ensure_grad(h, st);
@@ -896,7 +958,11 @@ pss_status pss_backward_grad(pss_handle* h, const float* grad_out, float* grad, 
     if (rc != PSS_OK) return rc;
     const bool sorted = h->batch_emitted && want_sorted(h, h->last_nnz * (int64_t)h->dp.J);
     h->last_path = sorted ? PSS_PATH_SORTED : PSS_PATH_ATOMIC;
-    if (sorted) {
+    if (sorted && h->deterministic && !h->circ && window_reduce_ok(h->dp, dg)) {
+        PSS_TRY(cudaMemsetAsync(grad, 0, sizeof(float) * (size_t)h->dp.M, st));
+        if ((rc = sorted_window(h, dg, staged, false, grad, st)) != PSS_OK) return rc;
+        if ((rc = grad_release(h, staged, st)) != PSS_OK) return rc;
+    } else if (sorted) {
         const int64_t saved = h->accum;
         h->accum = PSS_ACCUM_F64;
         rc = ensure_grad(h, st);

@@ -84,6 +84,7 @@ struct SortedBuffers {
     uint32_t* q_row;              // nnz output rows b*T + t written by the forward
     unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j), grouped by x
     unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets
+    float* bnd;                   // window reduce: boundary records, 64 floats per task
     // counting sort (R <= kCountSortMaxR)
     uint32_t* ccnt;               // R counts per bucket (zero between sorts)
     uint32_t* start;              // R + 1 bucket starts
@@ -117,6 +118,21 @@ cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t 
                               const Touched& touched, int sm_count, cudaStream_t st);
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
                                  const DevParams& p, double* g, int sm_count, cudaStream_t st);
+// Window reduce (see pss_sorted.cu): run sums go into each task's sliding
+// element window; every element's gradient is stored once into gexp (fp32,
+// zero where the batch adds nothing; the caller zero-fills it), in a fixed
+// order of additions.  Serves 32-element chunks tiling the rows (Z = 32,
+// d % 32 == 0, 16-byte aligned upstream gradient) when the array does not
+// wrap.
+struct WindowSink {
+    float* gexp;    // gradient out, M elements
+    float* bnd;     // window_records(npairs) records of 64 floats
+};
+bool window_reduce_ok(const DevParams& p, const float* gout);
+int64_t window_records(int64_t npairs);
+cudaError_t launch_window_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                                 const DevParams& p, const WindowSink& ws, int sm_count,
+                                 cudaStream_t st);
 
 // Kernel launchers (return the CUDA launch error).  `grid_cap` bounds the
 // grid of grid-stride kernels; 0 lets the launcher decide.

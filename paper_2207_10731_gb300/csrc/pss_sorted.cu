@@ -984,11 +984,28 @@ __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;\n" :: "n"(N) : "memory");
 }
 
-__global__ void __launch_bounds__(kThreads)
+// Where the staged reduce puts each run's sum (SINK):
+//   kSinkF64   added into the fp64 gradient accumulator g (red.global.add.f64);
+//   kSinkOnce  added into the task's ELEMENT WINDOW: the runs of a task come in
+//              ascending bucket order, so the 32 elements [wb, wb + 32) that
+//              lane z holds (element wb + z) slide forward; an element that
+//              leaves the window has all of the task's contributions.  If no
+//              other task can add to it (no bucket of the task before or after
+//              this one reaches it), its gradient is final and is stored once
+//              into ws.gexp (fp32).  Otherwise its partial sum goes to the
+//              task's boundary record (bnd[task][0..32): the window of its
+//              first bucket, [32..64): of its last), and k_window_combine
+//              stores it.  Every element's additions then happen in a fixed
+//              order, and nothing is added atomically.
+constexpr int kSinkF64 = 0;
+constexpr int kSinkOnce = 1;
+
+template <int SINK>
+__global__ void __launch_bounds__(kThreads, 4)
 k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int64_t G, uint32_t smask,
-               double* __restrict__ g) {
+               double* __restrict__ g, WindowSink ws) {
     pdl_prologue();
     __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
     __shared__ unsigned long long s_ent[kWarps][kAPiece];
@@ -1001,8 +1018,45 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
     constexpr unsigned long long kNone = (unsigned long long)kBad << 32;
     const uint64_t pol = l2_evict_first();
     float sum = 0.f, comp = 0.f;
+    // window sink: lane z holds element wb + z; the task's head boundary ends
+    // at hb_end, its tail boundary starts at tb_start; hx and tx are the first
+    // elements of its first and last buckets
+    int64_t wb = 0, hb_end = 0, tb_start = 0, hx = 0, tx = 0, task = 0;
+    float acc = 0.f, accc = 0.f;
+    auto finalize = [&](int lim) {   // the window's first lim elements are done
+        if (lane < lim) {
+            const int64_t e = wb + lane;
+            const float v = acc - accc;
+            if (e < hb_end || e >= tb_start) {
+                float* rec = ws.bnd + task * 64;
+                if (e < hx + 32) rec[e - hx] = v;
+                else rec[32 + (e - tx)] = v;
+            } else if (v != 0.f) {
+                ws.gexp[e] = v;
+            }
+        }
+    };
     auto flush = [&](uint32_t x) {
-        if (sum != 0.f) red_add_f64(g + (int64_t)x * G + lane, widen(sum));
+        if (SINK == kSinkF64) {
+            if (sum != 0.f) red_add_f64(g + (int64_t)x * G + lane, widen(sum));
+        } else {
+            const int64_t xb = (int64_t)x * G;
+            const int64_t sh = xb - wb;           // >= 0: buckets ascend
+            if (sh > 0) {
+                finalize(sh < 32 ? (int)sh : 32);
+                if (sh >= 32) {
+                    acc = accc = 0.f;
+                } else {
+                    const float a2 = __shfl_down_sync(0xffffffffu, acc, (int)sh);
+                    const float c2 = __shfl_down_sync(0xffffffffu, accc, (int)sh);
+                    const bool in = lane + (int)sh < 32;
+                    acc = in ? a2 : 0.f;
+                    accc = in ? c2 : 0.f;
+                }
+                wb = xb;
+            }
+            kahan_add(acc, accc, sum - comp);
+        }
         sum = comp = 0.f;
     };
     uint32_t nstart = 0;   // distinct buckets: entries whose bucket differs from the one before
@@ -1037,7 +1091,18 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         for (int st = 0; st < kAD - 1; ++st) issue(st);
         sum = comp = 0.f;
         uint32_t cur = (uint32_t)(ent[0] >> 32);
-        nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
+        const uint32_t xprev = (e0 > 0) ? (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) : kBad;
+        nstart += (e0 == 0 || xprev != cur) ? 1u : 0u;
+        if (SINK != kSinkF64) {
+            task = t;
+            hx = (int64_t)cur * G;
+            tx = (int64_t)(uint32_t)(ent[n - 1] >> 32) * G;
+            hb_end = (e0 > 0) ? (int64_t)xprev * G + 32 : 0;
+            tb_start = (e0 + n < total) ? (int64_t)(uint32_t)(__ldg(sorted_e + e0 + n) >> 32) * G
+                                        : INT64_MAX;
+            wb = hx;
+            acc = accc = 0.f;
+        }
         for (int st = 0; st < nst; ++st) {
             issue(st + kAD - 1);
             cp_async_wait<kAD - 1>();
@@ -1080,10 +1145,81 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
             __syncwarp();
         }
         flush(cur);
+        if (SINK != kSinkF64) finalize(32);
         cp_async_wait<0>();
         __syncwarp();
     }
     if (lane == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
+}
+
+// The boundary elements of the window reduce.  Between task j - 1 and task j
+// the elements [G*x_first(j), G*x_last(j-1) + 32) got partial sums from both
+// (and from more tasks when one bucket fills several).  One warp per task
+// boundary j, lane z on element e = G*x_first(j) + z: if e lies there and not
+// also past the next boundary, this warp owns e.  The tasks that hold e are
+// j, j - 1, ... down to the first that does not: the warp loads the bounds of
+// 32 tasks at a time (one per lane), each lane counts its tasks from them,
+// then loads their partials with independent loads and adds them in task
+// order (j first) in fp64, and stores the sum into ws.gexp.
+__global__ void __launch_bounds__(kThreads)
+k_window_combine(const unsigned long long* __restrict__ sorted_e,
+                 const unsigned long long* __restrict__ stats, int64_t npairs, int64_t G,
+                 WindowSink ws) {
+    pdl_prologue();
+    const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
+    const int64_t ntasks = (total + kAPiece - 1) / kAPiece;
+    const int lane = threadIdx.x & 31;
+    auto xat = [&](int64_t i) { return (int64_t)(uint32_t)(__ldg(sorted_e + i) >> 32) * G; };
+    auto xlast = [&](int64_t k) {
+        return xat(((k + 1) * kAPiece < total ? (k + 1) * kAPiece : total) - 1);
+    };
+    for (int64_t j = 1 + (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5); j < ntasks;
+         j += (int64_t)gridDim.x * kWarps) {
+        const int64_t xfj = xat(j * kAPiece);
+        const int64_t xlp = xat(j * kAPiece - 1);
+        const int64_t xfn = (j + 1 < ntasks) ? xat((j + 1) * kAPiece) : INT64_MAX;
+        const int64_t e = xfj + lane;
+        // shared with task j - 1, and no later boundary owns it
+        bool open = e < xlp + 32 && e < xfn;
+        if (!__any_sync(0xffffffffu, open)) continue;
+        double tot = 0.0;
+        for (int64_t kb = j; kb >= 0 && __any_sync(0xffffffffu, open); kb -= 32) {
+            // lane i: bounds of task kb - i
+            const int64_t kl = kb - lane;
+            const int64_t xfk = (kl >= 0) ? xat(kl * kAPiece) : INT64_MAX;
+            const int64_t xlk = (kl >= 0) ? xlast(kl) : 0;
+            // tasks kb, kb - 1, ... holding e: the first ncnt of this round
+            int ncnt = 0;
+            for (int i = 0; i < 32; ++i) {
+                const int64_t xf = __shfl_sync(0xffffffffu, xfk, i);
+                const int64_t xl = __shfl_sync(0xffffffffu, xlk, i);
+                const bool holds = open && e >= xf && e < xl + 32 && (e < xf + 32 || e >= xl);
+                if (holds) ++ncnt;
+                else open = false;
+            }
+            // their partials, loaded independently, added in task order
+            for (int i0 = 0; i0 < 32; i0 += 8) {
+                if (!__any_sync(0xffffffffu, i0 < ncnt)) break;
+                float p[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const int i = i0 + u;
+                    const int64_t xf = __shfl_sync(0xffffffffu, xfk, i);
+                    const int64_t xl = __shfl_sync(0xffffffffu, xlk, i);
+                    p[u] = 0.f;
+                    if (i < ncnt) {
+                        const float* rec = ws.bnd + (kb - i) * 64;
+                        p[u] = (e < xf + 32) ? rec[e - xf] : rec[32 + (e - xl)];
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                    if (i0 + u < ncnt) tot += widen(p[u]);
+            }
+        }
+        const float v = narrow(tot);
+        if (v != 0.f && e < xlp + 32 && e < xfn) ws.gexp[e] = v;
+    }
 }
 
 template <int KE, bool ZDIV, bool JPOW2>
@@ -1243,14 +1379,37 @@ cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t 
                     touched);
 }
 
+bool window_reduce_ok(const DevParams& p, const float* gout) {
+    return p.Z == 32 && p.d % 32 == 0 && (((uintptr_t)gout & 15u) == 0);
+}
+
+int64_t window_records(int64_t npairs) { return (npairs + kAPiece - 1) / kAPiece; }
+
+cudaError_t launch_window_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
+                                 const DevParams& p, const WindowSink& ws, int sm_count,
+                                 cudaStream_t st) {
+    if (!window_reduce_ok(p, gout)) return cudaErrorInvalidValue;
+    const int64_t ntasks = window_records(npairs);   // upper bound
+    const int64_t blocks = (ntasks + kWarps - 1) / kWarps;
+    int grid = grid_for(k_async_reduce<kSinkOnce>, sm_count, blocks);
+    cudaError_t e = launch_k(k_async_reduce<kSinkOnce>, dim3(grid), dim3(kThreads), 0, st,
+                             sb.sorted_e, sb.stats, npairs, gout, p.G, p.smask,
+                             (double*)nullptr, ws);
+    if (e != cudaSuccess) return e;
+    grid = grid_for(k_window_combine, sm_count, blocks);
+    return launch_k(k_window_combine, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e,
+                    (const unsigned long long*)sb.stats, npairs, p.G, ws);
+}
+
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
                                  const DevParams& p, double* g, int sm_count, cudaStream_t st) {
     // 32-element chunks tiling the rows: asynchronous shared-memory staging
-    if (p.Z == 32 && p.d % 32 == 0 && (((uintptr_t)gout & 15u) == 0)) {
+    if (window_reduce_ok(p, gout)) {
         const int64_t ntasks = (npairs + kAPiece - 1) / kAPiece;   // upper bound
-        const int grid = grid_for(k_async_reduce, sm_count, (ntasks + kWarps - 1) / kWarps);
-        return launch_k(k_async_reduce, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e, sb.stats,
-                        npairs, gout, p.G, p.smask, g);
+        const int grid = grid_for(k_async_reduce<kSinkF64>, sm_count,
+                                  (ntasks + kWarps - 1) / kWarps);
+        return launch_k(k_async_reduce<kSinkF64>, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e,
+                        sb.stats, npairs, gout, p.G, p.smask, g, WindowSink{});
     }
     // blocks of 32+ elements: one warp per task, one element per lane
     if (p.L >= 32) {

@@ -140,7 +140,7 @@ def test_grad_parity(case, path):
     h.close()
 
 
-@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("path", ["atomic", "sorted", "sorted-deterministic"])
 def test_grad_single_hot_id_and_repeated_backward(path):
     # Every bag of every table holds id 0, so each table's J buckets collect
     # all B contributions (the most skewed batch there is); B is not a
@@ -149,6 +149,11 @@ def test_grad_single_hot_id_and_repeated_backward(path):
     w = wl.make_workload("tb", B=5003)
     w.indices[:] = 0
     h, o = gu.make_pair(w)
+    if path == "sorted-deterministic":
+        # every bucket's run fills about a thousand reduce tasks: the window
+        # reduce's boundary combine adds them all up
+        h.set_option(binding.OPT_DETERMINISTIC, 1)
+        path = "sorted"
     h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
     h.forward(*_batch_cuda(w), w.B)
     go = gu.cuda(w.grad_out)
@@ -412,7 +417,8 @@ def _sub_batch(w, rows):
 
 
 SWEEP = ([(lm, "auto") for lm in (18, 20, 22, 24, 26, 28, 30, 32, 33)] +
-         [(lm, "atomic") for lm in (28, 30, 32, 33)])
+         [(lm, "atomic") for lm in (28, 30, 32, 33)] +
+         [(lm, "deterministic") for lm in (20, 26, 30)])
 
 
 @pytest.mark.parametrize("logM,path", SWEEP, ids=[f"2^{lm}-{p}" for lm, p in SWEEP])
@@ -426,7 +432,9 @@ def test_compression_sweep(logM, path):
     M = 1 << logM
     w = wl.make_workload("sweep", M=M)
     h, o = gu.make_pair(w)
-    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    if path == "deterministic":
+        h.set_option(binding.OPT_DETERMINISTIC, 1)
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS.get(path, binding.PATH_AUTO))
     idx, off = _batch_cuda(w)
     out = h.forward(idx, off, w.B)
     rng = np.random.default_rng(logM)
