@@ -328,6 +328,9 @@ def _config_extra(args, w):
         extra["mode"] = "forward only (inference): hash + gather + sum-pool, no backward"
     if args.signed:
         extra["signed_hash"] = True
+    if args.deterministic:
+        extra["deterministic"] = ("stable radix sort and window reduce: run-to-run identical bits "
+                                  "(PSS_OPT_DETERMINISTIC)")
     if args.ids == "uniform":
         extra["ids"] = "uniform over each table"
     return extra
@@ -421,6 +424,8 @@ def run_gpu(args):
     h.set_option(binding.OPT_ACCUM, binding.ACCUM_F32 if args.accum == "f32" else binding.ACCUM_F64)
     if args.signed:
         h.set_option(binding.OPT_SIGNED, 1)
+    if args.deterministic:
+        h.set_option(binding.OPT_DETERMINISTIC, 1)
     # forward-only: no backward follows, so the forward emits nothing for one
     h.set_option(binding.OPT_BACKWARD_PATH,
                  binding.PATH_ATOMIC if args.forward_only else
@@ -621,6 +626,8 @@ def main(argv=None):
     ap.add_argument("--forward-only", action="store_true",
                     help="time the forward (inference) alone")
     ap.add_argument("--signed", action="store_true", help="signed hashing (PSS_OPT_SIGNED)")
+    ap.add_argument("--deterministic", action="store_true",
+                    help="run-to-run identical bits on the sorted path (PSS_OPT_DETERMINISTIC)")
     ap.add_argument("--ids", choices=["workload", "uniform"], default="workload",
                     help="id distribution: the workload's own (Zipf for the Criteo shapes) or "
                          "uniform over each table")
