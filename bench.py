@@ -62,6 +62,14 @@ def _host():
                 model = m.group(1).strip()
                 break
         if model is None:
+            try:
+                out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+                m = re.search(r"^Model name:\s*(.+)$", out, flags=re.M)
+                if m:
+                    model = m.group(1).strip()
+            except (OSError, subprocess.SubprocessError):
+                pass
+        if model is None:
             impl = re.search(r"^CPU implementer\s*:\s*(\S+)", info, flags=re.M)
             part = re.search(r"^CPU part\s*:\s*(\S+)", info, flags=re.M)
             if impl and part:
@@ -238,6 +246,21 @@ def _algorithmic_bytes(w: wl.Workload):
     }
 
 
+def _touched_elements(h, dbatches, L, torch):
+    """Mean number of distinct elements of M that a batch's blocks cover (the
+    touched update reads and writes only these): the union of the intervals
+    [loc, loc + L) over the batch's locations, from the library's own hash."""
+    tot = 0
+    for i, o, _ in dbatches:
+        nb = (o.numel() - 1) // h.T
+        loc = h.compute_locations(i, o, nb)
+        u = torch.unique(loc[loc >= 0])
+        if u.numel():
+            tot += int(torch.clamp(torch.diff(u), max=L).sum().item()) + L
+    torch.cuda.synchronize()
+    return tot / max(1, len(dbatches))
+
+
 def _step_roofline(ab, step_s, hbm_peak, l2, forward_only, array_in_l2):
     """The step's bound: HBM time of its streamed bytes against L2 time of its
     shared-array gathers and adds (when the array is L2-resident), the larger
@@ -319,6 +342,14 @@ def _shape_overrides(args):
     return over
 
 
+def _workload_desc(args, w):
+    """The named workload's description with the batch and M actually run."""
+    desc = re.sub(r"batch \d+", f"batch {w.B}", WORKLOAD_DESC[args.workload])
+    if args.M is not None:
+        desc = re.sub(r"M=[0-9.]+M[i]? fp32( \(\d+ MB\))?|M chosen by --M", f"M={w.M} fp32", desc)
+    return desc
+
+
 def _config_extra(args, w):
     """Config keys that differ from the named workload's defaults."""
     extra = {}
@@ -376,7 +407,7 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64+f32",
         "data": "synthetic",
-        "config": dict({"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B, "seq_len": 1,
+        "config": dict({"workload": _workload_desc(args, w), "global_batch": w.B, "seq_len": 1,
                         "parallelism": "single host thread"}, **_config_extra(args, w)),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "host": _host(), "sample": sample},
@@ -526,12 +557,21 @@ def run_gpu(args):
     # gradient: 16 bytes per element) fits in L2
     l2_size = getattr(props, "L2_cache_size", 0) or (126 << 20)
     array_in_l2 = 16 * w.M <= l2_size // 2
+    # the optimizer pass visits only the touched blocks when M exceeds the
+    # batch's pairs * L (the library's automatic rule for the update mode)
+    L = min(w.Z, w.d)
+    touched_elems = None
+    if (not args.forward_only and rank == 0
+            and w.M > min(nnz_per_step) * (-(-w.d // w.Z)) * L):
+        touched_elems = _touched_elements(h, dbatches, L, torch)
 
     if rank == 0:
         clocks = sampler.summary(wall0, wall2) if sampler else None
         value = lookups / (elapsed_ms / 1e3)
         peak, peak_kind = _peaks()
         ab = _algorithmic_bytes(w)
+        if touched_elems is not None:
+            ab["update"] = (16 if w.opt == "adagrad" else 8) * touched_elems
         # dominant kernel with an algorithmic byte count (sort passes are pure
         # implementation overhead and have none)
         cands = {k: v for k, v in prof.items() if k in ab} or {"forward": (1, float("nan"))}
@@ -544,6 +584,9 @@ def run_gpu(args):
                  "unit": "GB/s", "frac": achieved / peak, "traffic": _traffic(dom, args.workload),
                  "peak_kind": peak_kind, "algorithmic_bytes_per_launch": bytes_dom,
                  "avg_launch_ms": avg_s * 1e3}
+        if dom == "update" and touched_elems is not None:
+            kroof["note"] = (f"touched update: {touched_elems:.0f} distinct elements of M per batch "
+                             "(union of the batch's blocks), each read and written once")
         if dom == "forward" and array_in_l2 and l2:
             # the forward's block gathers from the L2-resident array take
             # longer at the measured L2 gather rate than its HBM streams
@@ -570,7 +613,7 @@ def run_gpu(args):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": WORKLOAD_DESC[args.workload], "global_batch": w.B * world,
+            "config": {"workload": _workload_desc(args, w), "global_batch": w.B * world,
                        "seq_len": 1,
                        "parallelism": "independent replicas" if world > 1 else "single GPU",
                        "grad_accumulator": args.accum,
