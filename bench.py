@@ -350,6 +350,20 @@ def _workload_desc(args, w):
     return desc
 
 
+def _sort_desc(h, binding, args):
+    """How the sorted path grouped the pairs in the timed steps."""
+    info = h.info()
+    if info["last_path"] != binding.PATH_SORTED:
+        return {}
+    if args.deterministic:
+        return {"sort": "stable radix sort of all pairs"}
+    if info["last_collision_rate"] < 0:
+        return {"sort": "segment-local: pairs grouped by location within 8192-pair segments"}
+    return {"sort": ("counting sort of all pairs" if info["R"] <= (1 << 22) else
+                     "radix sort of all pairs"),
+            "collision_rate": info["last_collision_rate"]}
+
+
 def _config_extra(args, w):
     """Config keys that differ from the named workload's defaults."""
     extra = {}
@@ -457,6 +471,8 @@ def run_gpu(args):
         h.set_option(binding.OPT_SIGNED, 1)
     if args.deterministic:
         h.set_option(binding.OPT_DETERMINISTIC, 1)
+    h.set_option(binding.OPT_SORT_SCOPE, {"auto": binding.SORT_AUTO, "global": binding.SORT_GLOBAL,
+                                          "local": binding.SORT_LOCAL}[args.sort])
     # forward-only: no backward follows, so the forward emits nothing for one
     h.set_option(binding.OPT_BACKWARD_PATH,
                  binding.PATH_ATOMIC if args.forward_only else
@@ -618,6 +634,7 @@ def run_gpu(args):
                        "parallelism": "independent replicas" if world > 1 else "single GPU",
                        "grad_accumulator": args.accum,
                        "backward_path": ["auto", "atomic", "sorted"][h.info()["last_path"]],
+                       **_sort_desc(h, binding, args),
                        "l2": (f"inputs larger than L2: {args.rotate}-batch rotation, "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB output and "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB upstream gradient per step"),
@@ -669,6 +686,9 @@ def main(argv=None):
     ap.add_argument("--forward-only", action="store_true",
                     help="time the forward (inference) alone")
     ap.add_argument("--signed", action="store_true", help="signed hashing (PSS_OPT_SIGNED)")
+    ap.add_argument("--sort", choices=["auto", "global", "local"], default="auto",
+                    help="sorted path: one sort over all pairs, the segment-local sort, or the "
+                         "library's choice (PSS_OPT_SORT_SCOPE)")
     ap.add_argument("--deterministic", action="store_true",
                     help="run-to-run identical bits on the sorted path (PSS_OPT_DETERMINISTIC)")
     ap.add_argument("--ids", choices=["workload", "uniform"], default="workload",

@@ -146,7 +146,20 @@ typedef enum {
      * a location follows the GPU's scheduling (the sum is within the same
      * bound, but low-order bits may differ between runs).  Above 2^22 block
      * starts the radix sort is always used.  The atomic path is not affected. */
-    PSS_OPT_DETERMINISTIC = 9
+    PSS_OPT_DETERMINISTIC = 9,
+    /* How the sorted path (when not deterministic) groups the pairs by
+     * location.  PSS_SORT_GLOBAL: one sort of all pairs (counting sort up to
+     * 2^22 block starts, radix sort above).  PSS_SORT_LOCAL: within segments
+     * of 8192 consecutive pairs only, one run per location and segment (the
+     * runs of a location meet in the fp64 accumulator); no per-location
+     * state, any R; needs chunks that tile the rows (Z = 32, d a multiple of
+     * 32, 16-byte aligned upstream gradient), else the global sort runs.
+     * PSS_SORT_AUTO (default): local where it is served and either R > 2^22
+     * or the batch has at most PSS_SORT_LOCAL_MAX_PAIRS_PER_START pairs per
+     * block start (few repeats to merge across segments); global otherwise.
+     * After a local pass pss_info's last_collision_rate is -1 (no distinct
+     * locations are counted). */
+    PSS_OPT_SORT_SCOPE = 10
 } pss_option;
 
 
@@ -155,6 +168,8 @@ enum { PSS_ACCUM_F64 = 0, PSS_ACCUM_F32 = 1 };
 
 enum { PSS_PATH_AUTO = 0, PSS_PATH_ATOMIC = 1, PSS_PATH_SORTED = 2 };
 enum { PSS_UPDATE_AUTO = 0, PSS_UPDATE_DENSE = 1, PSS_UPDATE_TOUCHED = 2 };
+enum { PSS_SORT_AUTO = 0, PSS_SORT_GLOBAL = 1, PSS_SORT_LOCAL = 2 };
+#define PSS_SORT_LOCAL_MAX_PAIRS_PER_START 4
 
 /* Kernel ids for pss_get_profile. */
 typedef enum {

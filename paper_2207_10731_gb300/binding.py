@@ -27,9 +27,11 @@ OPT_SIGNED = 6
 OPT_CIRCULAR = 7
 OPT_SORT_DIGIT_BITS = 8
 OPT_DETERMINISTIC = 9
+OPT_SORT_SCOPE = 10
 ACCUM_F64, ACCUM_F32 = 0, 1
 PATH_AUTO, PATH_ATOMIC, PATH_SORTED = 0, 1, 2
 UPDATE_AUTO, UPDATE_DENSE, UPDATE_TOUCHED = 0, 1, 2
+SORT_AUTO, SORT_GLOBAL, SORT_LOCAL = 0, 1, 2
 K_LOCATIONS, K_FORWARD, K_SCATTER, K_UPDATE, K_SORT, K_REDUCE, K_MISC = range(7)
 KERNEL_NAMES = ["locations", "forward", "scatter", "update", "sort", "reduce", "misc"]
 

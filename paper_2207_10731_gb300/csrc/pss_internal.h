@@ -85,6 +85,7 @@ struct SortedBuffers {
     unsigned long long* sorted_e; // nnz*J entries (x << 32 | row*J + j), grouped by x
     unsigned long long* stats;    // [0] valid pairs, [1] distinct buckets
     float* bnd;                   // window reduce: boundary records, 64 floats per task
+    uint32_t* segn;               // local sort: valid pairs of each segment
     // counting sort (R <= kCountSortMaxR)
     uint32_t* ccnt;               // R counts per bucket (zero between sorts)
     uint32_t* start;              // R + 1 bucket starts
@@ -116,8 +117,19 @@ cudaError_t launch_radix_sort(const SortedBuffers& sb, int64_t npairs, int J, ui
 // Touched bitmap / list of the buckets of the forward's pairs.
 cudaError_t launch_mark_pairs(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
                               const Touched& touched, int sm_count, cudaStream_t st);
+// Segment-local sort (see pss_sorted.cu): the valid entries of each segment of
+// consecutive pairs grouped by bucket inside the segment's range of sorted_e,
+// their number in segn[local_segments(npairs)].  Serves the shapes of the
+// staged reduce (local_sort_ok) with R < 2^32 - 1; any R, no per-bucket state.
+int64_t local_segments(int64_t npairs);
+bool local_sort_ok(const DevParams& p, const float* gout);
+cudaError_t launch_sort_local(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
+                              int sm_count, cudaStream_t st);
+// Reduce of the sorted entries into g (fp64).  `local`: the entries come from
+// the segment-local sort (one run per bucket and segment).
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                                 const DevParams& p, double* g, int sm_count, cudaStream_t st);
+                                 const DevParams& p, double* g, bool local, int sm_count,
+                                 cudaStream_t st);
 // Window reduce (see pss_sorted.cu): run sums go into each task's sliding
 // element window; every element's gradient is stored once into gexp (fp32,
 // zero where the batch adds nothing; the caller zero-fills it), in a fixed

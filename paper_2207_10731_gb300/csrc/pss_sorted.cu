@@ -326,6 +326,120 @@ k_sort_scatter(const uint32_t* __restrict__ pair_x, int64_t npairs, const uint32
 }
 
 // ---------------------------------------------------------------------------
+// Segment-local sort.  The pairs are cut into segments of kLS consecutive
+// pairs, and each segment's valid entries are grouped by bucket inside the
+// segment's own range of sorted_e, [s*kLS, s*kLS + segn[s]): no counter per
+// bucket, no scan over all R buckets, no global atomics.  A bucket that occurs
+// in several segments then has one run in each; the reduce adds every run's
+// sum into the fp64 accumulator, so each element receives the same sum,
+// grouped differently.  Consecutive pairs are consecutive ids of one table,
+// so a segment merges the repeats of the table's hot ids (under Zipf ids the
+// ones that would otherwise queue reductions on one address).
+//
+// Within a segment: every thread inserts its pairs into a shared-memory hash
+// table (bucket -> count; each pair's rank among the segment's pairs of its
+// bucket), the slot counts are scanned in a fixed slot order, and a pair goes
+// to its slot's start plus its rank.  Which pair of a bucket comes first
+// follows the order of the shared-memory atomics.
+constexpr int kLSLog2 = 13;
+constexpr int kLS = 1 << kLSLog2;                 // pairs per segment (8192)
+constexpr int kLSThreads = 1024;
+constexpr int kLSPer = kLS / kLSThreads;          // pairs per thread
+constexpr int kLSLog2Slots = kLSLog2 + 1;         // load factor <= 1/2
+constexpr int kLSSlots = 1 << kLSLog2Slots;
+constexpr int kLSSlotsPer = kLSSlots / kLSThreads;
+static_assert(kLS <= 65536 && kLSSlots <= 65536, "slot and rank are packed in 16 bits each");
+static_assert(kLSThreads == kScanThreads, "the local sort scans with block_exclusive_scan");
+
+__device__ __forceinline__ uint32_t local_insert(uint32_t* s_key, uint32_t* s_val, uint32_t x) {
+    uint32_t h = (x * 0x9e3779b1u) >> (32 - kLSLog2Slots);
+    for (int probe = 0; probe < kLSSlots; ++probe) {
+        const uint32_t prev = atomicCAS(s_key + h, kEmpty, x);
+        if (prev == kEmpty || prev == x) break;
+        h = (h + 1u) & (uint32_t)(kLSSlots - 1);
+    }
+    return h | (atomicAdd(s_val + h, 1u) << 16);
+}
+
+// sorted_e[s*kLS + pos] = x << 32 | row*J + j for the valid pairs of segment
+// s, grouped by x; segn[s] = the segment's number of valid pairs.
+template <bool SG>
+__global__ void __launch_bounds__(kLSThreads, 1)
+k_sort_local(const uint32_t* __restrict__ pair_x, int64_t npairs,
+             const uint32_t* __restrict__ q_row, int J, int log2J,
+             unsigned long long* __restrict__ sorted_e, uint32_t* __restrict__ segn) {
+    pdl_prologue();
+    extern __shared__ __align__(16) uint32_t s_ls[];
+    uint32_t* s_key = s_ls;
+    uint32_t* s_val = s_ls + kLSSlots;
+    __shared__ uint32_t s_warp[33];
+    const int tid = threadIdx.x;
+#pragma unroll
+    for (int k = 0; k < kLSSlotsPer; ++k) {
+        s_key[k * kLSThreads + tid] = kEmpty;
+        s_val[k * kLSThreads + tid] = 0u;
+    }
+    const int64_t nseg = (npairs + kLS - 1) / kLS;
+    for (int64_t seg = blockIdx.x; seg < nseg; seg += gridDim.x) {
+        const int64_t p0 = seg * kLS;
+        uint32_t x[kLSPer], e[kLSPer], hr[kLSPer];
+#pragma unroll
+        for (int i = 0; i < kLSPer; ++i) {
+            const int64_t p = p0 + i * kLSThreads + tid;
+            x[i] = (p < npairs) ? __ldg(pair_x + p) : kBad;
+        }
+#pragma unroll
+        for (int i = 0; i < kLSPer; ++i) {
+            const uint32_t pp = (uint32_t)(p0 + i * kLSThreads + tid);   // npairs < 2^32 here
+            const uint32_t q = (log2J >= 0) ? (pp >> log2J) : pp / (uint32_t)J;
+            e[i] = pp - q * (uint32_t)J;
+            if (x[i] != kBad) {
+                e[i] += __ldg(q_row + q) * (uint32_t)J;
+                if (SG) {
+                    // signed hashing: the sign moves to bit 31 of the entry's low word
+                    e[i] |= x[i] & 0x80000000u;
+                    x[i] &= 0x7fffffffu;
+                }
+            }
+        }
+        __syncthreads();   // the previous segment's table is clear
+#pragma unroll
+        for (int i = 0; i < kLSPer; ++i)
+            hr[i] = (x[i] != kBad) ? local_insert(s_key, s_val, x[i]) : 0u;
+        __syncthreads();
+        // slot starts: exclusive prefix of the counts in the order (thread,
+        // k) over the slots tid + k*kLSThreads that thread tid owns
+        uint32_t c[kLSSlotsPer], own = 0u;
+#pragma unroll
+        for (int k = 0; k < kLSSlotsPer; ++k) {
+            c[k] = s_val[k * kLSThreads + tid];
+            own += c[k];
+        }
+        uint32_t total;
+        uint32_t run = block_exclusive_scan(own, s_warp, &total);
+#pragma unroll
+        for (int k = 0; k < kLSSlotsPer; ++k) {
+            s_val[k * kLSThreads + tid] = run;
+            run += c[k];
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kLSPer; ++i) {
+            if (x[i] == kBad) continue;
+            const uint32_t pos = s_val[hr[i] & 0xffffu] + (hr[i] >> 16);
+            sorted_e[p0 + pos] = ((unsigned long long)x[i] << 32) | e[i];
+        }
+        if (tid == 0) segn[seg] = total;
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < kLSSlotsPer; ++k) {
+            s_key[k * kLSThreads + tid] = kEmpty;
+            s_val[k * kLSThreads + tid] = 0u;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Stable LSD radix sort of the pairs by bucket x.
 //
 // The keys are the bucket indices (at most 32 bits); the sort makes P passes of
@@ -1005,12 +1119,19 @@ __global__ void __launch_bounds__(kThreads, 4)
 k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int64_t G, uint32_t smask,
-               double* __restrict__ g, WindowSink ws) {
+               double* __restrict__ g, WindowSink ws, const uint32_t* __restrict__ segn) {
     pdl_prologue();
     __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
     __shared__ unsigned long long s_ent[kWarps][kAPiece];
-    const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
-    const int64_t ntasks = (total + kAPiece - 1) / kAPiece;
+    // segn: the segment-local layout (k_sort_local), kLS / kAPiece tasks per
+    // segment, each cut at the segment's valid entries; otherwise one sorted
+    // run of stats[0] valid entries
+    constexpr int kPieces = kLS / kAPiece;
+    const bool local = segn != nullptr;
+    const int64_t total =
+        local ? npairs : (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
+    const int64_t ntasks =
+        local ? ((npairs + kLS - 1) / kLS) * kPieces : (total + kAPiece - 1) / kAPiece;
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     unsigned long long* ent = s_ent[warp];
@@ -1061,8 +1182,19 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
     };
     uint32_t nstart = 0;   // distinct buckets: entries whose bucket differs from the one before
     for (int64_t t = (int64_t)blockIdx.x * kWarps + warp; t < ntasks; t += wstride) {
-        const int64_t e0 = t * kAPiece;
-        const int n = (int)((e0 + kAPiece < total) ? kAPiece : total - e0);
+        int64_t e0;
+        int n;
+        if (local) {
+            const int64_t s = t / kPieces;
+            const int k = (int)(t - s * kPieces);
+            const int left = (int)__ldg(segn + s) - k * kAPiece;
+            if (left <= 0) continue;
+            e0 = s * kLS + (int64_t)k * kAPiece;
+            n = left < kAPiece ? left : kAPiece;
+        } else {
+            e0 = t * kAPiece;
+            n = (int)((e0 + kAPiece < total) ? kAPiece : total - e0);
+        }
 #pragma unroll
         for (int h = 0; h < kAPiece; h += 32)
             ent[h + lane] = (h + lane < n) ? ld_once_u64(sorted_e + e0 + h + lane, pol) : kNone;
@@ -1091,7 +1223,8 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         for (int st = 0; st < kAD - 1; ++st) issue(st);
         sum = comp = 0.f;
         uint32_t cur = (uint32_t)(ent[0] >> 32);
-        const uint32_t xprev = (e0 > 0) ? (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) : kBad;
+        const uint32_t xprev =
+            (e0 > 0 && !local) ? (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) : kBad;
         nstart += (e0 == 0 || xprev != cur) ? 1u : 0u;
         if (SINK != kSinkF64) {
             task = t;
@@ -1149,7 +1282,8 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         cp_async_wait<0>();
         __syncwarp();
     }
-    if (lane == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
+    // (the local layout's runs are per segment: no distinct-bucket count)
+    if (lane == 0 && nstart && !local) atomicAdd(stats + 1, (unsigned long long)nstart);
 }
 
 // The boundary elements of the window reduce.  Between task j - 1 and task j
@@ -1394,15 +1528,40 @@ cudaError_t launch_window_reduce(const SortedBuffers& sb, int64_t npairs, const 
     int grid = grid_for(k_async_reduce<kSinkOnce>, sm_count, blocks);
     cudaError_t e = launch_k(k_async_reduce<kSinkOnce>, dim3(grid), dim3(kThreads), 0, st,
                              sb.sorted_e, sb.stats, npairs, gout, p.G, p.smask,
-                             (double*)nullptr, ws);
+                             (double*)nullptr, ws, (const uint32_t*)nullptr);
     if (e != cudaSuccess) return e;
     grid = grid_for(k_window_combine, sm_count, blocks);
     return launch_k(k_window_combine, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e,
                     (const unsigned long long*)sb.stats, npairs, p.G, ws);
 }
 
+int64_t local_segments(int64_t npairs) { return (npairs + kLS - 1) / kLS; }
+
+bool local_sort_ok(const DevParams& p, const float* gout) { return window_reduce_ok(p, gout); }
+
+cudaError_t launch_sort_local(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
+                              int sm_count, cudaStream_t st) {
+    if (npairs <= 0) return cudaSuccess;
+    const int log2J = ((J & (J - 1)) == 0) ? ceil_log2(J) : -1;
+    const size_t smem = sizeof(uint32_t) * 2 * (size_t)kLSSlots;
+    auto kern = smask ? k_sort_local<true> : k_sort_local<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kLSThreads, smem) !=
+            cudaSuccess || per_sm < 1)
+        per_sm = 1;
+    const int64_t nseg = local_segments(npairs);
+    const int grid = (int)(nseg < (int64_t)sm_count * per_sm ? nseg : (int64_t)sm_count * per_sm);
+    return launch_k(kern, dim3(grid), dim3(kLSThreads), smem, st, sb.pair_x, npairs, sb.q_row, J,
+                    log2J, sb.sorted_e, sb.segn);
+}
+
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                                 const DevParams& p, double* g, int sm_count, cudaStream_t st) {
+                                 const DevParams& p, double* g, bool local, int sm_count,
+                                 cudaStream_t st) {
+    if (local && !window_reduce_ok(p, gout)) return cudaErrorInvalidValue;
     // 32-element chunks tiling the rows: asynchronous shared-memory staging
     if (window_reduce_ok(p, gout)) {
         // 3 CTAs per SM (measured at the Criteo-TB shape: 0.170 ms against
@@ -1412,7 +1571,8 @@ cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const 
         int grid = grid_for(k_async_reduce<kSinkF64>, sm_count, (ntasks + kWarps - 1) / kWarps);
         if (grid > 3 * sm_count) grid = 3 * sm_count;
         return launch_k(k_async_reduce<kSinkF64>, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e,
-                        sb.stats, npairs, gout, p.G, p.smask, g, WindowSink{});
+                        sb.stats, npairs, gout, p.G, p.smask, g, WindowSink{},
+                        local ? (const uint32_t*)sb.segn : (const uint32_t*)nullptr);
     }
     // blocks of 32+ elements: one warp per task, one element per lane
     if (p.L >= 32) {

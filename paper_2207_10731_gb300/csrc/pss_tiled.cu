@@ -27,6 +27,7 @@ namespace {
 constexpr int kU = 4;            // ids in flight per group (the multi-id path sums them as a tree)
 static_assert(kU == 4, "the multi-id forward sums kU = 4 values per round as a tree");
 constexpr int kBagsPerGroup = 16;
+constexpr int kUB = 4;           // bags in flight per group in the forward's one-id path
 
 template <typename XT>
 struct Invalid;
@@ -254,10 +255,10 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
             warp_stage_bags<XT, SG>(p, idx, t, card, s_off, nb, s_x, err, pair_x, q_row,
                                 (uint32_t)(b0 * p.T + t), lane);
             float* orow0 = obase + gb0 * ostride;
-            for (int bb0 = gb0; bb0 < gb1; bb0 += kU) {
-                VT v[kU][KC];
+            for (int bb0 = gb0; bb0 < gb1; bb0 += kUB) {
+                VT v[kUB][KC];
 #pragma unroll
-                for (int u = 0; u < kU; ++u) {
+                for (int u = 0; u < kUB; ++u) {
                     const int bb = bb0 + u;
 #pragma unroll
                     for (int k = 0; k < KC; ++k) {
@@ -270,7 +271,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                     }
                 }
 #pragma unroll
-                for (int u = 0; u < kU; ++u) {
+                for (int u = 0; u < kUB; ++u) {
                     if (bb0 + u >= gb1) break;
 #pragma unroll
                     for (int k = 0; k < KC; ++k)

@@ -119,12 +119,25 @@ def test_forward_dyadic_bit_exact(name, B):
 PATHS = {"auto": binding.PATH_AUTO, "atomic": binding.PATH_ATOMIC, "sorted": binding.PATH_SORTED}
 
 
-@pytest.mark.parametrize("path", list(PATHS))
+def _set_path(h, path):
+    """Select a backward path by name: "sorted" leaves the sort scope automatic,
+    "sorted-local" and "sorted-global" force the segment-local sort (where
+    the chunks tile the rows) or one sort over all pairs.  Returns the PATH_*
+    value."""
+    if path in ("sorted-global", "sorted-local"):
+        h.set_option(binding.OPT_SORT_SCOPE,
+                     binding.SORT_GLOBAL if path == "sorted-global" else binding.SORT_LOCAL)
+        path = "sorted"
+    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    return PATHS[path]
+
+
+@pytest.mark.parametrize("path", list(PATHS) + ["sorted-global", "sorted-local"])
 @pytest.mark.parametrize("case", FWD_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
 def test_grad_parity(case, path):
     w = _wl(case)
     h, o = gu.make_pair(w)
-    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    want = _set_path(h, path)
     h.forward(*_batch_cuda(w), w.B)
     g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
     ref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
@@ -136,7 +149,7 @@ def test_grad_parity(case, path):
     mass = float((lengths.T * rows).sum())
     assert abs(g.astype(np.float64).sum() - mass) <= 1e-5 * A.sum() + 1e-6
     if path != "auto":
-        assert h.info()["last_path"] == PATHS[path]
+        assert h.info()["last_path"] == want
     h.close()
 
 
@@ -204,7 +217,7 @@ def _run_step(w, h, o, wcur, Gcur, batch):
     return gu.host(wg), (gu.host(Gg) if Gg is not None else None), w2, G2, g32, A
 
 
-@pytest.mark.parametrize("path", list(PATHS))
+@pytest.mark.parametrize("path", list(PATHS) + ["sorted-global", "sorted-local"])
 @pytest.mark.parametrize("case", STEP_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
 def test_step_parity_three_steps(case, path):
     case = dict(case)
@@ -216,7 +229,7 @@ def test_step_parity_three_steps(case, path):
     if lr:
         w.lr = lr
     h, o = gu.make_pair(w)
-    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    _set_path(h, path)
     wcur = w.w0.copy()
     Gcur = np.zeros(w.M, dtype=np.float32)
     cfg = wl.CONFIGS[case["name"]]
@@ -279,11 +292,18 @@ def test_dense_and_touched_updates_identical_on_both_paths():
 
 
 def test_sorted_path_reports_collision_rate():
-    # rho = 1 - distinct blocks / (ids * chunks), from the sorted pass's counters
+    # rho = 1 - distinct blocks / (ids * chunks), from the global sort's
+    # counters; the segment-local sort counts no distinct blocks (-1)
     t = gu.torch()
     w = wl.make_workload("tb", B=4096)
     h, o = gu.make_pair(w)
     h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    h.set_option(binding.OPT_SORT_SCOPE, binding.SORT_LOCAL)
+    h.forward(*_batch_cuda(w), w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    t.cuda.synchronize()
+    assert h.info()["last_collision_rate"] == -1.0
+    h.set_option(binding.OPT_SORT_SCOPE, binding.SORT_GLOBAL)
     h.forward(*_batch_cuda(w), w.B)
     h.backward_update(gu.cuda(w.grad_out), w.lr)
     t.cuda.synchronize()
@@ -418,6 +438,7 @@ def _sub_batch(w, rows):
 
 SWEEP = ([(lm, "auto") for lm in (18, 20, 22, 24, 26, 28, 30, 32, 33)] +
          [(lm, "atomic") for lm in (28, 30, 32, 33)] +
+         [(lm, "global") for lm in (24, 30)] +
          [(lm, "deterministic") for lm in (20, 26, 30)])
 
 
@@ -426,14 +447,17 @@ def test_compression_sweep(logM, path):
     """Criteo-TB shape with M from 2^18 to 2^33 fp32 (1 MB .. 32 GB).  Up to
     2^26 everything is compared; above, sampled rows and sampled elements
     (touched and untouched) are compared with the oracle evaluated one by one.
-    AUTO takes the sorted path here (a radix sort of up to three passes); the
-    atomic path is forced at the large sizes too."""
+    AUTO takes the sorted path here (the segment-local sort; "global" sorts
+    all pairs at once: counting sort at 2^24, radix sort at 2^30); the atomic
+    path is forced at the large sizes too."""
     t = gu.torch()
     M = 1 << logM
     w = wl.make_workload("sweep", M=M)
     h, o = gu.make_pair(w)
     if path == "deterministic":
         h.set_option(binding.OPT_DETERMINISTIC, 1)
+    if path == "global":
+        h.set_option(binding.OPT_SORT_SCOPE, binding.SORT_GLOBAL)
     h.set_option(binding.OPT_BACKWARD_PATH, PATHS.get(path, binding.PATH_AUTO))
     idx, off = _batch_cuda(w)
     out = h.forward(idx, off, w.B)
@@ -602,11 +626,11 @@ def _signed_pair(w, path):
     h, o_u = gu.make_pair(w)
     o = OraclePSS(w.cards, d=w.d, M=w.M, Z=w.Z, G=w.G, seed=w.seed, signed=True)
     h.set_option(binding.OPT_SIGNED, 1)
-    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    _set_path(h, path)
     return h, o, o_u
 
 
-@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("path", ["atomic", "sorted-global", "sorted-local"])
 @pytest.mark.parametrize("case", SIGNED_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
 def test_signed_hashing_forward_and_grad_parity(case, path):
     w = _wl(case)
@@ -622,7 +646,7 @@ def test_signed_hashing_forward_and_grad_parity(case, path):
     gref = o.grad(w.indices, w.offsets, w.B, w.grad_out)
     A = o_u.grad(w.indices, w.offsets, w.B, np.abs(w.grad_out))
     gu.check_grad(g, gref, A, what="signed grad")
-    assert h.info()["last_path"] == PATHS[path]
+    assert h.info()["last_path"] == PATHS[path.split("-")[0]]
     h.close()
 
 
@@ -689,13 +713,13 @@ def _circ_pair(w, path, signed=False):
     h.set_option(binding.OPT_CIRCULAR, 1)
     if signed:
         h.set_option(binding.OPT_SIGNED, 1)
-    h.set_option(binding.OPT_BACKWARD_PATH, PATHS[path])
+    _set_path(h, path)
     h.set_weights(gu.cuda(w.w0))      # (re)load: refreshes the mirror of M[0 .. L)
     return h, o, o_abs
 
 
 @pytest.mark.parametrize("signed", [False, True])
-@pytest.mark.parametrize("path", ["atomic", "sorted"])
+@pytest.mark.parametrize("path", ["atomic", "sorted-global", "sorted-local"])
 @pytest.mark.parametrize("case", CIRC_CASES, ids=lambda c: "-".join(f"{k}{v}" for k, v in c.items()))
 def test_circular_forward_and_grad_parity(case, path, signed):
     w = _wl(case)
@@ -872,6 +896,89 @@ def test_out_of_range_ids_are_skipped_and_reported(path):
     h.close()
 
 
+@pytest.mark.parametrize("path", ["sorted-local", "sorted-global"])
+def test_out_of_range_ids_in_local_segments(path):
+    # 32-float chunks (the segment-local sort): bad ids scattered over several
+    # 8192-pair segments, one segment with many; each segment's valid entries
+    # are counted and the rest of its range is never read
+    w = wl.make_workload("tb", B=3001)
+    idx = w.indices.copy()
+    rng = np.random.default_rng(5)
+    bad = np.concatenate([rng.choice(idx.shape[0], 40, replace=False),
+                          np.arange(5000, 5600)])
+    idx[bad] = -1
+    idx[bad[:20]] = 1 << 40
+    h, o = gu.make_pair(w)
+    _set_path(h, path)
+    h.forward(gu.cuda(idx), gu.cuda(w.offsets), w.B)
+    st, first = h.get_error()
+    assert st == binding.PSS_ERR_INDEX_RANGE and first == int(bad.min())
+    g = gu.host(h.backward_grad(gu.cuda(w.grad_out)))
+    gref = o.grad(idx, w.offsets, w.B, w.grad_out)
+    A = o.grad(idx, w.offsets, w.B, np.abs(w.grad_out))
+    gu.check_grad(g, gref, A)
+    h.close()
+
+
+@pytest.mark.parametrize("name,B", [("tb", 3001), ("multihot", 777)])
+@pytest.mark.parametrize("opt", ["sgd", "adagrad"])
+def test_local_sort_step_dyadic_bit_exact(name, B, opt):
+    # dyadic inputs: every partial sum is exact, so the segment-local
+    # grouping gives the oracle's bits whatever the order of its additions
+    w = wl.make_workload(name, B=B, grad="dyadic", w0="dyadic")
+    w.lr = 0.125
+    h, o = gu.make_pair(w, opt=opt)
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    h.set_option(binding.OPT_SORT_SCOPE, binding.SORT_LOCAL)
+    h.forward(*_batch_cuda(w), w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    wg, Gg = h.get_state()
+    w2, G2, _ = o.step(w.w0, np.zeros(w.M, np.float32), w.indices, w.offsets, w.B, w.grad_out,
+                       opt, w.lr, w.eps)
+    np.testing.assert_array_equal(gu.host(wg), w2)
+    if opt == "adagrad":
+        np.testing.assert_array_equal(gu.host(Gg), G2)
+    assert h.info()["last_collision_rate"] == -1.0     # the local sort ran
+    h.close()
+
+
+def test_sort_scope_option_rules():
+    w = wl.make_workload("tiny")
+    h, _ = gu.make_pair(w)
+    assert h.get_option(binding.OPT_SORT_SCOPE) == binding.SORT_AUTO
+    for bad in (-1, 3):
+        with pytest.raises(binding.PSSError):
+            h.set_option(binding.OPT_SORT_SCOPE, bad)
+    for v in (binding.SORT_GLOBAL, binding.SORT_LOCAL, binding.SORT_AUTO):
+        h.set_option(binding.OPT_SORT_SCOPE, v)
+        assert h.get_option(binding.OPT_SORT_SCOPE) == v
+    h.close()
+
+
+@pytest.mark.parametrize("name,B,local", [("tb", 1024, True), ("tb", 65536, False),
+                                          ("microbench", 10240, True), ("tiny", 256, False)])
+def test_sort_scope_auto_rule(name, B, local):
+    # AUTO: local where the chunks tile the rows and the batch has at most
+    # 4 pairs per block start (R > 2^22 aside); the collision rate tells
+    # which ran (-1 after a local pass)
+    t = gu.torch()
+    w = wl.make_workload(name, B=B)
+    h, _ = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    idx, off = _batch_cuda(w)
+    go = gu.cuda(w.grad_out)
+    for _ in range(2):        # the global sort's counts reach the host by the next call
+        h.forward(idx, off, w.B)
+        h.backward_update(go, w.lr)
+    t.cuda.synchronize()
+    h.forward(idx, off, w.B)
+    h.backward_update(go, w.lr)
+    pairs = w.indices.shape[0] * (-(-w.d // w.Z))
+    assert (pairs <= 4 * h.info()["R"]) == local or name == "tiny"
+    assert (h.info()["last_collision_rate"] == -1.0) == local
+    h.close()
+
+
 def test_malformed_offsets_reported():
     w = wl.make_workload("tiny")
     off = w.offsets.copy()
@@ -947,6 +1054,20 @@ def test_profile_and_launch_counts():
     h.forward(idx, off, w.B)
     h.backward_update(go, w.lr)
     assert h.info()["kernel_launches"] - before == 9
+    h.close()
+    # 32-float chunks: forward, segment-local sort, reduce, update
+    w = wl.make_workload("tb", B=2048)
+    h, _ = gu.make_pair(w)
+    h.set_option(binding.OPT_BACKWARD_PATH, binding.PATH_SORTED)
+    h.set_option(binding.OPT_SORT_SCOPE, binding.SORT_LOCAL)
+    h.set_option(binding.OPT_UPDATE_MODE, binding.UPDATE_DENSE)
+    idx, off = _batch_cuda(w)
+    h.forward(idx, off, w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    before = h.info()["kernel_launches"]
+    h.forward(idx, off, w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    assert h.info()["kernel_launches"] - before == 4
     h.close()
 
 
