@@ -782,8 +782,8 @@ static pss_status sort_pairs(pss_handle* h, bool touch, bool local, cudaStream_t
         if (touch)
             PSS_TRY(launch_mark_pairs(h->sb, npairs, h->dp.smask, h->touched, h->sm_count, st));
     } else {
-        // ccnt is zero here: it is zeroed when allocated, and every sort's slot
-        // scatter counts each bucket back down by exactly what its count added
+        // ccnt is zero here: it is zeroed when allocated, and every sort's scan
+        // returns the counters it has read to zero
         pss_status rc0 = ensure_counting(h, st);
         if (rc0 != PSS_OK) return rc0;
         LaunchScope ls(h, PSS_K_SORT, st, 5);

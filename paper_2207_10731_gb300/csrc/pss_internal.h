@@ -102,8 +102,9 @@ struct SortedBuffers {
 constexpr int64_t kCountSortMaxR = int64_t(1) << 22;
 int64_t sorted_scan_blocks(int64_t R);
 // Counting sort: per-bucket counts of the valid pairs (ccnt must be zero on
-// entry), their scan (with `touched`, also the list / bitmap of non-empty
-// buckets), and the slot scatter into sorted_e (which returns ccnt to zero).
+// entry), their scan into the bucket starts (which returns ccnt to zero; with
+// `touched`, also the list / bitmap of non-empty buckets), and the slot
+// scatter into sorted_e (which advances each start to its bucket's end).
 cudaError_t launch_sorted_count(const SortedBuffers& sb, int64_t npairs, uint32_t smask,
                                 int sm_count, cudaStream_t st);
 cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched* touched,
