@@ -786,7 +786,7 @@ static pss_status sort_pairs(pss_handle* h, bool touch, bool local, cudaStream_t
         // returns the counters it has read to zero
         pss_status rc0 = ensure_counting(h, st);
         if (rc0 != PSS_OK) return rc0;
-        LaunchScope ls(h, PSS_K_SORT, st, 5);
+        LaunchScope ls(h, PSS_K_SORT, st, 4);
         PSS_TRY(launch_sorted_count(h->sb, npairs, h->dp.smask, h->sm_count, st));
         PSS_TRY(launch_sorted_scan(h->sb, (int64_t)h->dp.R, touch ? &h->touched : nullptr, st));
         PSS_TRY(launch_sorted_scatter(h->sb, npairs, h->dp.J, h->dp.smask, h->sm_count, st));

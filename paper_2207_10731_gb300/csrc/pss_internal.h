@@ -89,7 +89,7 @@ struct SortedBuffers {
     // counting sort (R <= kCountSortMaxR)
     uint32_t* ccnt;               // R counts per bucket (zero between sorts)
     uint32_t* start;              // R + 1 bucket starts
-    uint32_t* bsum;               // per scan chunk: entries, then their exclusive prefix
+    uint32_t* bsum;               // per scan chunk: entries
     uint32_t* bnz;                // per scan chunk: non-empty buckets
     // radix sort
     unsigned long long* tmp_e;    // nnz*J entries: the other buffer of the radix passes

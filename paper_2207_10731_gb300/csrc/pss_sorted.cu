@@ -69,7 +69,7 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* s
 
 // ---------------------------------------------------------------------------
 // Counting sort by bucket (the default when R <= kCountSortMaxR): a count of
-// every bucket, a scan of the counts (three kernels), and a slot scatter.
+// every bucket, a scan of the counts (two kernels), and a slot scatter.
 // Every bucket has its own counter, so the entries come out grouped by bucket;
 // their order inside a bucket depends on the GPU's scheduling.
 // Per chunk of kScanChunk counters: entries and non-empty buckets.
@@ -94,54 +94,27 @@ k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict_
     if (threadIdx.x == 0) bnz[blockIdx.x] = tot;
 }
 
-// Exclusive scans of the chunk sums and of the chunk non-empty counts (one
-// block).  stats[0] = valid pairs; stats[1] is cleared (the reduce counts the
-// distinct buckets); the number of non-empty buckets is the length of the
-// touched list when one is built.
-__global__ void __launch_bounds__(kScanThreads)
-k_scan_top(uint32_t* __restrict__ bsum, uint32_t* __restrict__ bnz, int64_t nblk,
-           unsigned long long* __restrict__ stats, unsigned long long* __restrict__ touched_count) {
-    pdl_prologue();
-    __shared__ uint32_t s_warp[33];
-    __shared__ uint32_t s_carry[2];
-    if (threadIdx.x < 2) s_carry[threadIdx.x] = 0;
-    __syncthreads();
-    for (int64_t b0 = 0; b0 < nblk; b0 += kScanThreads) {
-        const int64_t b = b0 + threadIdx.x;
-        const bool in = b < nblk;
-        const uint32_t v = in ? bsum[b] : 0u;
-        const uint32_t z = in ? bnz[b] : 0u;
-        uint32_t tot_v, tot_z;
-        const uint32_t ex_v = block_exclusive_scan(v, s_warp, &tot_v);
-        const uint32_t ex_z = block_exclusive_scan(z, s_warp, &tot_z);
-        const uint32_t cv = s_carry[0], cz = s_carry[1];
-        if (in) {
-            bsum[b] = cv + ex_v;
-            bnz[b] = cz + ex_z;
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            s_carry[0] = cv + tot_v;
-            s_carry[1] = cz + tot_z;
-        }
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-        stats[0] = s_carry[0];
-        stats[1] = 0;
-        if (touched_count) *touched_count = s_carry[1];
-    }
-}
-
 // start[x] = exclusive prefix of cnt; start[R] = total; cnt returns to zero
-// for the next sort's count.  With a touched list, the non-empty buckets are
-// listed in order and their bits set.
+// for the next sort's count.  Each block first adds up the chunk sums of the
+// blocks before it (a few hundred values).  The last block writes stats[0] =
+// valid pairs and clears stats[1] (the reduce counts the distinct buckets).
+// With a touched list, the non-empty buckets are listed in order and their
+// bits set, and the last block writes the list's length.
 __global__ void __launch_bounds__(kScanThreads)
 k_scan_apply(uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __restrict__ bsum,
-             const uint32_t* __restrict__ bnz, uint32_t* __restrict__ start, Touched tc) {
+             const uint32_t* __restrict__ bnz, uint32_t* __restrict__ start, Touched tc,
+             unsigned long long* __restrict__ stats) {
     pdl_prologue();
     __shared__ uint32_t s_warp[33];
     const int64_t base = (int64_t)blockIdx.x * kScanChunk;
+    uint32_t pv = 0u, pz = 0u;
+    for (int64_t b = threadIdx.x; b < (int64_t)blockIdx.x; b += kScanThreads) {
+        pv += bsum[b];
+        pz += bnz[b];
+    }
+    uint32_t pre_v, pre_z;
+    block_exclusive_scan(pv, s_warp, &pre_v);
+    block_exclusive_scan(pz, s_warp, &pre_z);
     uint32_t c[kScanPerThread];
     uint32_t sum = 0, nz = 0;
 #pragma unroll
@@ -152,9 +125,14 @@ k_scan_apply(uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __restrict__
         sum += c[i];
         nz += (c[i] != 0u);
     }
-    uint32_t tot;
-    uint32_t run = bsum[blockIdx.x] + block_exclusive_scan(sum, s_warp, &tot);
-    uint32_t zrun = bnz[blockIdx.x] + block_exclusive_scan(nz, s_warp, &tot);
+    uint32_t tot_v, tot_z;
+    uint32_t run = pre_v + block_exclusive_scan(sum, s_warp, &tot_v);
+    uint32_t zrun = pre_z + block_exclusive_scan(nz, s_warp, &tot_z);
+    if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) {
+        stats[0] = pre_v + tot_v;
+        stats[1] = 0;
+        if (tc.count) *tc.count = pre_z + tot_z;
+    }
 #pragma unroll
     for (int i = 0; i < kScanPerThread; ++i) {
         const int64_t e = base + (int64_t)threadIdx.x * kScanPerThread + i;
@@ -1482,11 +1460,8 @@ cudaError_t launch_sorted_scan(const SortedBuffers& sb, int64_t R, const Touched
     cudaError_t e = launch_k(k_scan_reduce, dim3((unsigned)nblk), dim3(kScanThreads), 0, st,
                              sb.ccnt, R, sb.bsum, sb.bnz);
     if (e != cudaSuccess) return e;
-    e = launch_k(k_scan_top, dim3(1), dim3(kScanThreads), 0, st, sb.bsum, sb.bnz, nblk, sb.stats,
-                 tc.count);
-    if (e != cudaSuccess) return e;
     return launch_k(k_scan_apply, dim3((unsigned)nblk), dim3(kScanThreads), 0, st, sb.ccnt, R,
-                    sb.bsum, sb.bnz, sb.start, tc);
+                    sb.bsum, sb.bnz, sb.start, tc, sb.stats);
 }
 
 cudaError_t launch_sorted_scatter(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
