@@ -102,10 +102,15 @@ __device__ __forceinline__ void stage_buckets(const DevParams& p, const int64_t*
 
 // One VW-wide load of a staged block (bucket x, column offset z); with signed
 // hashing (SG) the bucket carries the sign in bit 31, applied to the value.
+// G < 2^31 (an int32 of the API): with 32-bit buckets the element index is
+// one 32 x 32 -> 64-bit multiply.
 template <bool SG, typename V, typename XT>
 __device__ __forceinline__ typename V::T gather(const float* __restrict__ w, uint64_t G, XT x, int z) {
-    if (!SG) return V::ldg(w + G * (uint64_t)x + z);
-    return sign_by(V::ldg(w + G * (uint64_t)(x & ~(XT)0x80000000u) + z), (uint32_t)x & 0x80000000u);
+    const XT xb = SG ? (x & ~(XT)0x80000000u) : x;
+    const uint64_t e = (sizeof(XT) == 4) ? (uint64_t)(uint32_t)G * (uint32_t)xb + (uint32_t)z
+                                         : G * (uint64_t)xb + (uint64_t)z;
+    if (!SG) return V::ldg(w + e);
+    return sign_by(V::ldg(w + e), (uint32_t)x & 0x80000000u);
 }
 
 // ---------------------------------------------------------------------------
@@ -306,21 +311,22 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                                        lane);
                 }
                 const int64_t qend = c < sw1 ? c : sw1;
-                for (int64_t qs = q; qs < qend; qs += (int64_t)kU * ng) {
+                // ids of the staged window by their 32-bit offset in it
+                const int i1 = (int)(qend - sw0);
+                for (int is = (int)(q - sw0); is < i1; is += kU * ng) {
                     VT v[kU][KC];
 #pragma unroll
                     for (int u = 0; u < kU; ++u) {
-                        const int64_t qq = qs + (int64_t)u * ng + g;
+                        const int ii = is + u * ng + g;
 #pragma unroll
                         for (int k = 0; k < KC; ++k) {
 #pragma unroll
                             for (int i = 0; i < VW; ++i) V::set(v[u][k], i, 0.f);
-                            if (qq < qend && col.v[k]) {
-                                const XT x = s_x[(int)(qq - sw0) * J + col.j[k]];
+                            if (ii < i1 && col.v[k]) {
+                                const XT x = s_x[ii * J + col.j[k]];
                                 if (x != Invalid<XT>::v) v[u][k] = gather<SG, V>(w, G, x, col.z[k]);
                             }
                         }
-                        if (qq < qend && q_row && lg == 0) q_row[qq] = row;
                     }
 #pragma unroll
                     for (int k = 0; k < KC; ++k)
@@ -333,6 +339,9 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                 }
                 q = qend;
             }
+            // the bag's ids' output row, one store per lane
+            if (q_row)
+                for (int64_t qq = a + lane; qq < c; qq += 32) q_row[qq] = row;
             for (int o = gs; o < 32; o <<= 1) {
 #pragma unroll
                 for (int k = 0; k < KC; ++k)
