@@ -24,8 +24,12 @@
 namespace pss {
 namespace {
 
-constexpr int kU = 4;            // ids in flight per group (the multi-id path sums them as a tree)
-static_assert(kU == 4, "the multi-id forward sums kU = 4 values per round as a tree");
+constexpr int kU = 4;            // ids in flight per group
+// ids in flight per group in the multi-id forward (4 or 8; measured on GB300
+// at the multi-hot shape: 8 took 0.398 ms per forward with spills and 0.381
+// at 3 CTAs per SM, against 0.334 ms with 4)
+constexpr int kUM = 4;
+static_assert(kUM == 4 || kUM == 8, "the multi-id forward sums 4 or 8 values per round as a tree");
 constexpr int kBagsPerGroup = 16;
 constexpr int kUB = 4;           // bags in flight per group in the forward's one-id path
 
@@ -289,8 +293,8 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
         }
 
         // general bags: the whole warp takes one bag at a time; its ng lane
-        // groups add ng consecutive ids of the bag in parallel, kU steps per
-        // round.  A round's kU values are summed as a tree and added to the
+        // groups add ng consecutive ids of the bag in parallel, kUM steps per
+        // round.  A round's kUM values are summed as a tree and added to the
         // running sum with compensation (Kahan); at the end of the bag the
         // groups' sums are merged the same way and group 0 stores the row.
         const int ng = 32 >> log2gs;
@@ -313,10 +317,10 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                 const int64_t qend = c < sw1 ? c : sw1;
                 // ids of the staged window by their 32-bit offset in it
                 const int i1 = (int)(qend - sw0);
-                for (int is = (int)(q - sw0); is < i1; is += kU * ng) {
-                    VT v[kU][KC];
+                for (int is = (int)(q - sw0); is < i1; is += kUM * ng) {
+                    VT v[kUM][KC];
 #pragma unroll
-                    for (int u = 0; u < kU; ++u) {
+                    for (int u = 0; u < kUM; ++u) {
                         const int ii = is + u * ng + g;
 #pragma unroll
                         for (int k = 0; k < KC; ++k) {
@@ -332,9 +336,12 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                     for (int k = 0; k < KC; ++k)
 #pragma unroll
                         for (int i = 0; i < VW; ++i) {
-                            const float s01 = V::get(v[0][k], i) + V::get(v[1][k], i);
-                            const float s23 = V::get(v[2][k], i) + V::get(v[3][k], i);
-                            kahan_add(acc[k][i], cmp[k][i], s01 + s23);
+                            float r = (V::get(v[0][k], i) + V::get(v[1][k], i)) +
+                                      (V::get(v[2][k], i) + V::get(v[3][k], i));
+                            if (kUM == 8)
+                                r += (V::get(v[kUM / 2][k], i) + V::get(v[kUM / 2 + 1][k], i)) +
+                                     (V::get(v[kUM - 2][k], i) + V::get(v[kUM - 1][k], i));
+                            kahan_add(acc[k][i], cmp[k][i], r);
                         }
                 }
                 q = qend;
