@@ -1309,6 +1309,8 @@ k_window_combine(const unsigned long long* __restrict__ sorted_e,
             // tasks kb, kb - 1, ... holding e: the first ncnt of this round
             int ncnt = 0;
             for (int i = 0; i < 32; ++i) {
+                // (most boundaries are shared by two tasks only)
+                if (!__any_sync(0xffffffffu, open)) break;
                 const int64_t xf = __shfl_sync(0xffffffffu, xfk, i);
                 const int64_t xl = __shfl_sync(0xffffffffu, xlk, i);
                 const bool holds = open && e >= xf && e < xl + 32 && (e < xf + 32 || e >= xl);
