@@ -473,6 +473,8 @@ def run_gpu(args):
         h.set_option(binding.OPT_DETERMINISTIC, 1)
     h.set_option(binding.OPT_SORT_SCOPE, {"auto": binding.SORT_AUTO, "global": binding.SORT_GLOBAL,
                                           "local": binding.SORT_LOCAL}[args.sort])
+    h.set_option(binding.OPT_UPDATE_MODE, {"auto": binding.UPDATE_AUTO, "dense": binding.UPDATE_DENSE,
+                                           "touched": binding.UPDATE_TOUCHED}[args.update])
     # forward-only: no backward follows, so the forward emits nothing for one
     h.set_option(binding.OPT_BACKWARD_PATH,
                  binding.PATH_ATOMIC if args.forward_only else
@@ -573,12 +575,12 @@ def run_gpu(args):
     # gradient: 16 bytes per element) fits in L2
     l2_size = getattr(props, "L2_cache_size", 0) or (126 << 20)
     array_in_l2 = 16 * w.M <= l2_size // 2
-    # the optimizer pass visits only the touched blocks when M exceeds the
-    # batch's pairs * L (the library's automatic rule for the update mode)
+    # the optimizer pass visits only the touched blocks when the library chose
+    # its touched update
     L = min(w.Z, w.d)
     touched_elems = None
     if (not args.forward_only and rank == 0
-            and w.M > min(nnz_per_step) * (-(-w.d // w.Z)) * L):
+            and h.info()["last_update"] == binding.UPDATE_TOUCHED):
         touched_elems = _touched_elements(h, dbatches, L, torch)
 
     if rank == 0:
@@ -635,6 +637,9 @@ def run_gpu(args):
                        "grad_accumulator": args.accum,
                        "backward_path": ["auto", "atomic", "sorted"][h.info()["last_path"]],
                        **_sort_desc(h, binding, args),
+                       **({} if args.forward_only else
+                          {"update": {binding.UPDATE_DENSE: "dense", binding.UPDATE_TOUCHED: "touched blocks"}
+                           .get(h.info()["last_update"], "SGD scattered into M")}),
                        "l2": (f"inputs larger than L2: {args.rotate}-batch rotation, "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB output and "
                               f"{w.B * w.T * w.d * 4 / 1e6:.0f} MB upstream gradient per step"),
@@ -686,6 +691,8 @@ def main(argv=None):
     ap.add_argument("--forward-only", action="store_true",
                     help="time the forward (inference) alone")
     ap.add_argument("--signed", action="store_true", help="signed hashing (PSS_OPT_SIGNED)")
+    ap.add_argument("--update", choices=["auto", "dense", "touched"], default="auto",
+                    help="how the optimizer pass visits M (PSS_OPT_UPDATE_MODE)")
     ap.add_argument("--sort", choices=["auto", "global", "local"], default="auto",
                     help="sorted path: one sort over all pairs, the segment-local sort, or the "
                          "library's choice (PSS_OPT_SORT_SCOPE)")

@@ -96,7 +96,9 @@ typedef enum {
     PSS_OPT_BACKWARD_PATH = 1,
     /* How the Adagrad step visits M: every element (PSS_UPDATE_DENSE), only the
      * blocks the batch touched (PSS_UPDATE_TOUCHED), or chosen from M and the
-     * batch size (PSS_UPDATE_AUTO).  Results are identical. */
+     * batch size (PSS_UPDATE_AUTO: dense while 16 * M bytes fit in half the
+     * GPU's L2 or M <= nnz * J * L, touched otherwise).  Results are identical;
+     * pss_info's last_update says which pass ran. */
     PSS_OPT_UPDATE_MODE = 2,
     /* 1: record CUDA events around every kernel (read with pss_get_profile). */
     PSS_OPT_PROFILE = 3,
@@ -197,6 +199,9 @@ typedef struct {
     uint64_t A2, B2;           /* sign-hash parameters derived from the seed */
     int64_t signed_hash;       /* PSS_OPT_SIGNED */
     int64_t circular;          /* PSS_OPT_CIRCULAR */
+    int64_t last_update;       /* optimizer pass of the last pss_backward_update:
+                                  PSS_UPDATE_DENSE, PSS_UPDATE_TOUCHED, or 0 (none yet,
+                                  or SGD with the fp32 accumulator, scattered into M) */
 } pss_info;
 
 /*

@@ -53,7 +53,7 @@ class PSSInfo(ctypes.Structure):
                 ("kernel_launches", ctypes.c_int64), ("last_path", ctypes.c_int64),
                 ("last_collision_rate", ctypes.c_double), ("A2", ctypes.c_uint64),
                 ("B2", ctypes.c_uint64), ("signed_hash", ctypes.c_int64),
-                ("circular", ctypes.c_int64)]
+                ("circular", ctypes.c_int64), ("last_update", ctypes.c_int64)]
 
 
 class PSSError(RuntimeError):

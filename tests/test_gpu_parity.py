@@ -942,6 +942,27 @@ def test_local_sort_step_dyadic_bit_exact(name, B, opt):
     h.close()
 
 
+@pytest.mark.parametrize("name,B,M,want", [("kaggle", 2048, None, "dense"), ("tb", 64, None, "dense"),
+                                            ("sweep", 1024, 1 << 25, "touched"),
+                                            ("sweep", 65536, 1 << 25, "dense")])
+def test_update_mode_auto_rule(name, B, M, want):
+    # AUTO: dense while 16 * M bytes fit in half the L2 or M <= pairs * L;
+    # the touched pass otherwise (pss_info.last_update says which ran)
+    t = gu.torch()
+    w = wl.make_workload(name, B=B, M=M)
+    h, _ = gu.make_pair(w)
+    h.forward(*_batch_cuda(w), w.B)
+    h.backward_update(gu.cuda(w.grad_out), w.lr)
+    t.cuda.synchronize()
+    l2 = t.cuda.get_device_properties(0).L2_cache_size
+    pairs_l = w.indices.shape[0] * (-(-w.d // w.Z)) * min(w.Z, w.d)
+    assert (want == "touched") == (16 * w.M > l2 // 2 and w.M > pairs_l)
+    assert h.info()["last_update"] == {"dense": binding.UPDATE_DENSE,
+                                       "touched": binding.UPDATE_TOUCHED}[want]
+    assert h.get_error() == (binding.PSS_OK, -1)
+    h.close()
+
+
 def test_sort_scope_option_rules():
     w = wl.make_workload("tiny")
     h, _ = gu.make_pair(w)
