@@ -171,7 +171,7 @@ enum { PSS_ACCUM_F64 = 0, PSS_ACCUM_F32 = 1 };
 enum { PSS_PATH_AUTO = 0, PSS_PATH_ATOMIC = 1, PSS_PATH_SORTED = 2 };
 enum { PSS_UPDATE_AUTO = 0, PSS_UPDATE_DENSE = 1, PSS_UPDATE_TOUCHED = 2 };
 enum { PSS_SORT_AUTO = 0, PSS_SORT_GLOBAL = 1, PSS_SORT_LOCAL = 2 };
-#define PSS_SORT_LOCAL_MAX_PAIRS_PER_START 4
+#define PSS_SORT_LOCAL_MAX_PAIRS_PER_START 3
 
 /* Kernel ids for pss_get_profile. */
 typedef enum {

@@ -844,11 +844,12 @@ static pss_status ensure_g32(pss_handle* h, cudaStream_t st) {
 // Segment-local or global sort (PSS_OPT_SORT_SCOPE).  The local sort saves
 // the global sort's per-bucket counters and atomics but leaves one run per
 // bucket and segment, each an fp64 reduction of a chunk into g: it pays
-// where few pairs share a block start (measured at the Criteo-TB shape:
-// 11 pairs per start, global 0.478 ms per step against local 0.495; paper
-// micro-benchmark shape, 1.7 per start: local 0.105 against 0.116), and
-// above 2^22 starts, where the global sort is the radix sort (M = 2^28:
-// local 1.20 against 1.31 ms).
+// where few pairs share a block start, and above 2^22 starts, where the
+// global sort is the radix sort.  Measured on GB300 (ms per step, global
+// against local): Criteo-TB shape at 1.4, 2.7, 4.1 and 11 pairs per start
+// 0.098/0.090, 0.152/0.153, 0.207/0.215, 0.465/0.495; paper micro-benchmark
+// shape (1.7) 0.110/0.105; M = 2^22 at 3.3 per start 0.275/0.274; M = 2^24
+// (1.6) 0.635/0.629; M = 2^28 (radix) 1.31/1.20.
 static bool use_local_sort(const pss_handle* h, int64_t npairs, const float* dgrad) {
     if (h->deterministic || h->sort_scope == PSS_SORT_GLOBAL || !local_sort_ok(h->dp, dgrad))
         return false;
