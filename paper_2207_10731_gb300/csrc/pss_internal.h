@@ -152,12 +152,14 @@ cudaError_t launch_window_reduce(const SortedBuffers& sb, int64_t npairs, const 
 cudaError_t launch_locations(const DevParams& p, const int64_t* idx, int64_t nnz,
                              const int64_t* off, int64_t B, int64_t* locs, DevError* err,
                              int sm_count, cudaStream_t st);
-// Forward; when pair_x / q_row are given it also writes every pair's bucket
-// and every id's output row for the sorted backward path.
+// Forward of the bags of batch rows [b_lo, b_hi) of every table (0 <= b_lo <
+// b_hi <= B; out, idx and off are the whole batch's); when pair_x / q_row are
+// given it also writes those bags' pairs' buckets and ids' output rows for the
+// sorted backward path.
 cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
-                           DevError* err, uint32_t* pair_x, uint32_t* q_row, int sm_count,
-                           cudaStream_t st);
+                           DevError* err, uint32_t* pair_x, uint32_t* q_row, int64_t b_lo,
+                           int64_t b_hi, int sm_count, cudaStream_t st);
 // Backward scatter into an fp32 target (scale applied to grad_out) or into an
 // fp64 accumulator (scale 1).
 cudaError_t launch_scatter(const DevParams& p, const RowLayout& lay, const int64_t* idx,

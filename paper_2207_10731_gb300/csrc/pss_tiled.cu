@@ -200,7 +200,7 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
                const int64_t* __restrict__ off, int64_t B, const float* __restrict__ w,
                float* __restrict__ out, DevError* err, uint32_t* __restrict__ pair_x,
                uint32_t* __restrict__ q_row, int log2gs, int wb,
-               int tiles_per_table) {
+               int tiles_per_table, int64_t b_lo, int64_t b_hi) {
     pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
@@ -225,8 +225,8 @@ k_forward_warp(DevParams p, const int64_t* __restrict__ idx, int64_t nnz,
          tile += (int64_t)gridDim.x * kWarps) {
         // ntiles < 2^31 (checked by the launcher): 32-bit division
         const int t = (int)((uint32_t)tile / (uint32_t)tiles_per_table);
-        const int64_t b0 = (tile - (int64_t)t * tiles_per_table) * wb;
-        const int nb = (int)((B - b0) < wb ? (B - b0) : wb);
+        const int64_t b0 = b_lo + (tile - (int64_t)t * tiles_per_table) * wb;
+        const int nb = (int)((b_hi - b0) < wb ? (b_hi - b0) : wb);
         const int64_t s0 = (int64_t)t * B + b0;
         float* obase = out + ((b0 * p.T) + t) * (int64_t)p.d;
         const int gb0 = min(g * bpg, nb);
@@ -497,7 +497,7 @@ size_t tile_smem(const TileGeom& g, const DevParams& p, size_t xbytes) {
 template <int VW, int KC, typename XT, bool SG>
 cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                      const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
-                     uint32_t* pair_x, uint32_t* q_row, int sm_count,
+                     uint32_t* pair_x, uint32_t* q_row, int64_t b_lo, int64_t b_hi, int sm_count,
                      cudaStream_t st) {
     // bags per warp tile: kU per lane group (kU loads in flight in the one-id
     // path) and at least 16.  Measured on GB300: 16-bag tiles beat 32 and 64
@@ -507,7 +507,7 @@ cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* id
     // need the kU per group (batch 32768: 0.026 against 0.036 ms).
     const int groups = 32 >> lay.log2gs;
     const int wb = groups * kU > 16 ? groups * kU : 16;
-    const int tpt = (int)((B + wb - 1) / wb);
+    const int tpt = (int)((b_hi - b_lo + wb - 1) / wb);
     const size_t smem = (size_t)kWarps * ((size_t)(wb + 1) * sizeof(int64_t) +
                                           (size_t)kWarpPairs * sizeof(XT));
     const int64_t ntiles = (int64_t)p.T * tpt;
@@ -515,7 +515,7 @@ cudaError_t fwd_inst(const DevParams& p, const RowLayout& lay, const int64_t* id
     const int grid = grid_for(k_forward_warp<VW, KC, XT, SG>, sm_count, (ntiles + kWarps - 1) / kWarps,
                               smem);
     return launch_k(k_forward_warp<VW, KC, XT, SG>, dim3(grid), dim3(kThreads), smem, st, p, idx, nnz,
-                    off, B, w, out, err, pair_x, q_row, lay.log2gs, wb, tpt);
+                    off, B, w, out, err, pair_x, q_row, lay.log2gs, wb, tpt, b_lo, b_hi);
 }
 
 template <int VW, int KC, typename XT, typename AT, bool TOUCH>
@@ -533,16 +533,17 @@ cudaError_t sc_inst(const DevParams& p, const RowLayout& lay, const int64_t* idx
 template <int VW, int KC>
 cudaError_t fwd_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, int64_t nnz,
                   const int64_t* off, int64_t B, const float* w, float* out, DevError* err,
-                  uint32_t* pair_x, uint32_t* q_row, int sm_count,
+                  uint32_t* pair_x, uint32_t* q_row, int64_t b_lo, int64_t b_hi, int sm_count,
                   cudaStream_t st) {
     if (p.R < 0xffffffffull)
         return p.smask ? fwd_inst<VW, KC, uint32_t, true>(p, lay, idx, nnz, off, B, w, out, err,
-                                                           pair_x, q_row, sm_count, st)
+                                                           pair_x, q_row, b_lo, b_hi, sm_count, st)
                        : fwd_inst<VW, KC, uint32_t, false>(p, lay, idx, nnz, off, B, w, out, err,
-                                                            pair_x, q_row, sm_count, st);
+                                                            pair_x, q_row, b_lo, b_hi, sm_count,
+                                                            st);
     // R >= 2^32: 64-bit buckets, never signed (signed hashing needs R < 2^31)
     return fwd_inst<VW, KC, uint64_t, false>(p, lay, idx, nnz, off, B, w, out, err, nullptr,
-                                             nullptr, sm_count, st);
+                                             nullptr, b_lo, b_hi, sm_count, st);
 }
 
 template <int VW, int KC, typename AT>
@@ -569,10 +570,12 @@ cudaError_t sc_x(const DevParams& p, const RowLayout& lay, const int64_t* idx, i
 
 cudaError_t launch_forward(const DevParams& p, const RowLayout& lay, const int64_t* idx,
                            int64_t nnz, const int64_t* off, int64_t B, const float* w, float* out,
-                           DevError* err, uint32_t* pair_x, uint32_t* q_row, int sm_count,
-                           cudaStream_t st) {
-#define PSS_FW(VW, KC) \
-    return fwd_x<VW, KC>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row, sm_count, st)
+                           DevError* err, uint32_t* pair_x, uint32_t* q_row, int64_t b_lo,
+                           int64_t b_hi, int sm_count, cudaStream_t st) {
+    if (b_lo < 0 || b_hi > B || b_lo >= b_hi) return cudaErrorInvalidValue;
+#define PSS_FW(VW, KC)                                                                        \
+    return fwd_x<VW, KC>(p, lay, idx, nnz, off, B, w, out, err, pair_x, q_row, b_lo, b_hi, \
+                         sm_count, st)
     if (lay.vw == 4) {
         switch (lay.kc) {
             case 1: PSS_FW(4, 1);

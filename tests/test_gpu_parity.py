@@ -803,10 +803,13 @@ def test_circular_option_rules():
 
 # --------------------------------------------------------------------------
 # host buffers through the same C-ABI calls (the end-to-end path)
-def test_host_buffers_match_device_buffers():
+# Criteo-TB batch 8192: 109 MB of pooled output, which the forward computes in
+# chunks of batch rows and downloads chunk by chunk into pinned host memory
+@pytest.mark.parametrize("name,B", [("kaggle", None), ("tb", 8192)])
+def test_host_buffers_match_device_buffers(name, B):
     # dyadic inputs: every sum is exact, so both paths must give the same bits
     t = gu.torch()
-    w = wl.make_workload("kaggle", grad="dyadic", w0="dyadic")
+    w = wl.make_workload(name, B=B, grad="dyadic", w0="dyadic")
     w.lr = 0.125
     h1, _ = gu.make_pair(w, opt="sgd")
     h2, _ = gu.make_pair(w, opt="sgd")
