@@ -926,8 +926,8 @@ static pss_status sorted_into64(pss_handle* h, const float* dgrad, bool staged, 
     if (rc != PSS_OK) return rc;
     {
         LaunchScope ls(h, PSS_K_REDUCE, st);
-        PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64, local, h->sm_count,
-                                     st));
+        PSS_TRY(launch_sorted_reduce(h->sb, npairs, dgrad, h->dp, h->g64, local,
+                                     !local && use_radix(h), h->sm_count, st));
     }
     return local ? PSS_OK : copy_stats(h, st);
 }

@@ -127,10 +127,12 @@ bool local_sort_ok(const DevParams& p, const float* gout);
 cudaError_t launch_sort_local(const SortedBuffers& sb, int64_t npairs, int J, uint32_t smask,
                               int sm_count, cudaStream_t st);
 // Reduce of the sorted entries into g (fp64).  `local`: the entries come from
-// the segment-local sort (one run per bucket and segment).
+// the segment-local sort (one run per bucket and segment).  `count_runs`: the
+// reduce counts the distinct buckets into stats[1] (the radix sort's entries;
+// the counting sort's scan counts them itself).
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                                 const DevParams& p, double* g, bool local, int sm_count,
-                                 cudaStream_t st);
+                                 const DevParams& p, double* g, bool local, bool count_runs,
+                                 int sm_count, cudaStream_t st);
 // Window reduce (see pss_sorted.cu): run sums go into each task's sliding
 // element window; every element's gradient is stored once into gexp (fp32,
 // zero where the batch adds nothing; the caller zero-fills it), in a fixed

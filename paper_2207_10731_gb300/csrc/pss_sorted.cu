@@ -18,7 +18,8 @@
 //               every run's sum once into the fp64 gradient accumulator
 //               g[G*x + z] -- one reduction per run and element instead of one
 //               per contribution, and no queue of reductions on a hot address.
-//               The reduce also counts the distinct buckets (stats[1]).
+//               The distinct buckets (stats[1]) come from the counting sort's
+//               scan, or, after a radix sort, from the reduce.
 // With the touched update, k_mark_pairs lists the touched blocks from pair_x.
 // The optimizer pass over g follows (pss_kernels.cu).
 #include <climits>
@@ -97,7 +98,7 @@ k_scan_reduce(const uint32_t* __restrict__ cnt, int64_t R, uint32_t* __restrict_
 // start[x] = exclusive prefix of cnt; start[R] = total; cnt returns to zero
 // for the next sort's count.  Each block first adds up the chunk sums of the
 // blocks before it (a few hundred values).  The last block writes stats[0] =
-// valid pairs and clears stats[1] (the reduce counts the distinct buckets).
+// valid pairs and stats[1] = distinct buckets (non-empty counters).
 // With a touched list, the non-empty buckets are listed in order and their
 // bits set, and the last block writes the list's length.
 __global__ void __launch_bounds__(kScanThreads)
@@ -130,7 +131,7 @@ k_scan_apply(uint32_t* __restrict__ cnt, int64_t R, const uint32_t* __restrict__
     uint32_t zrun = pre_z + block_exclusive_scan(nz, s_warp, &tot_z);
     if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) {
         stats[0] = pre_v + tot_v;
-        stats[1] = 0;
+        stats[1] = pre_z + tot_z;   // distinct buckets: the non-empty counters
         if (tc.count) *tc.count = pre_z + tot_z;
     }
 #pragma unroll
@@ -806,7 +807,7 @@ __global__ void __launch_bounds__(kThreads, (KC == 1) ? 4 : 1)
 k_range_reduce(const unsigned long long* __restrict__ sorted_e,
                unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int d, int Z, int J, int log2J, int L, int64_t G,
-               uint32_t smask, double* __restrict__ g, int log2gs) {
+               uint32_t smask, double* __restrict__ g, int log2gs, bool count_runs) {
     pdl_prologue();
     using V = Vec<VW>;
     using VT = typename V::T;
@@ -859,7 +860,8 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
         for (int u = 0; u < kRU; ++u) nxt[u] = (e0 + u < e1) ? __ldg(sorted_e + e0 + u) : kNone;
         uint32_t cur = (uint32_t)(nxt[0] >> 32);
-        nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
+        if (count_runs)
+            nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
         for (int64_t e = e0; e < e1; e += kRU) {
             uint32_t xs[kRU];
             VT v[kRU][KC];
@@ -937,7 +939,7 @@ k_range_reduce(const unsigned long long* __restrict__ sorted_e,
         }
         flush(cur);
     }
-    if (lg == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
+    if (count_runs && lg == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
 }
 
 // Reduce for blocks of at least 32 elements: one WARP per task of kPiece
@@ -955,7 +957,7 @@ __global__ void __launch_bounds__(kThreads)
 k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
                     unsigned long long* __restrict__ stats, int64_t npairs,
                     const float* __restrict__ gout, int d, int Z, int J, int log2J, int L,
-                    int64_t G, uint32_t smask, double* __restrict__ g) {
+                    int64_t G, uint32_t smask, double* __restrict__ g, bool count_runs) {
     pdl_prologue();
     __shared__ unsigned long long s_ent[kWarps][kPiece];
     const int64_t total = (int64_t)(stats[0] < (unsigned long long)npairs ? stats[0] : npairs);
@@ -986,7 +988,8 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
 #pragma unroll
         for (int k = 0; k < KE; ++k) s[k] = c[k] = 0.f;
         uint32_t cur = (uint32_t)(ent[0] >> 32);
-        nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
+        if (count_runs)
+            nstart += (e0 == 0 || (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) != cur) ? 1u : 0u;
         for (int b = 0; b < n; b += kWU) {
             uint32_t xs[kWU];
             float v[kWU][KE];
@@ -1037,7 +1040,7 @@ k_warp_range_reduce(const unsigned long long* __restrict__ sorted_e,
         flush(cur);
         __syncwarp();
     }
-    if (lane == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
+    if (count_runs && lane == 0 && nstart) atomicAdd(stats + 1, (unsigned long long)nstart);
 }
 
 // Reduce for 32-element chunks that tile the rows (Z = 32 dividing d): the
@@ -1103,7 +1106,8 @@ __global__ void __launch_bounds__(kThreads, 4)
 k_async_reduce(const unsigned long long* __restrict__ sorted_e,
                unsigned long long* __restrict__ stats, int64_t npairs,
                const float* __restrict__ gout, int64_t G, uint32_t smask,
-               double* __restrict__ g, WindowSink ws, const uint32_t* __restrict__ segn) {
+               double* __restrict__ g, WindowSink ws, const uint32_t* __restrict__ segn,
+               bool count_runs) {
     pdl_prologue();
     __shared__ __align__(16) float s_ring[kWarps][kAD][kAS][32];
     __shared__ unsigned long long s_ent[kWarps][kAPiece];
@@ -1207,8 +1211,12 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         for (int st = 0; st < kAD - 1; ++st) issue(st);
         sum = comp = 0.f;
         uint32_t cur = (uint32_t)(ent[0] >> 32);
-        const uint32_t xprev =
-            (e0 > 0 && !local) ? (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32) : kBad;
+        // the previous entry's bucket: the window's head boundary, and the count
+        // of distinct buckets when this pass makes it
+        const bool need_prev = (SINK != kSinkF64) || count_runs;
+        const uint32_t xprev = (e0 > 0 && !local && need_prev)
+                                   ? (uint32_t)(__ldg(sorted_e + e0 - 1) >> 32)
+                                   : kBad;
         nstart += (e0 == 0 || xprev != cur) ? 1u : 0u;
         if (SINK != kSinkF64) {
             task = t;
@@ -1267,7 +1275,7 @@ k_async_reduce(const unsigned long long* __restrict__ sorted_e,
         __syncwarp();
     }
     // (the local layout's runs are per segment: no distinct-bucket count)
-    if (lane == 0 && nstart && !local) atomicAdd(stats + 1, (unsigned long long)nstart);
+    if (count_runs && lane == 0 && nstart && !local) atomicAdd(stats + 1, (unsigned long long)nstart);
 }
 
 // The boundary elements of the window reduce.  Between task j - 1 and task j
@@ -1344,50 +1352,58 @@ k_window_combine(const unsigned long long* __restrict__ sorted_e,
 
 template <int KE, bool ZDIV, bool JPOW2>
 cudaError_t warp_reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                               const DevParams& p, double* g, int log2J, int sm_count,
-                               cudaStream_t st) {
+                               const DevParams& p, double* g, int log2J, bool count_runs,
+                               int sm_count, cudaStream_t st) {
     const int64_t ntasks = (npairs + kPiece - 1) / kPiece;   // upper bound
     const int grid = grid_for(k_warp_range_reduce<KE, ZDIV, JPOW2>, sm_count,
                               (ntasks + kWarps - 1) / kWarps);
     return launch_k(k_warp_range_reduce<KE, ZDIV, JPOW2>, dim3(grid), dim3(kThreads), 0, st,
-                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g);
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g,
+                    count_runs);
 }
 
 template <int KE>
 cudaError_t warp_reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                             const DevParams& p, double* g, int sm_count, cudaStream_t st) {
+                             const DevParams& p, double* g, bool count_runs, int sm_count,
+                             cudaStream_t st) {
     const int log2J = (p.J & (p.J - 1)) == 0 ? ceil_log2(p.J) : -1;
     if (p.d % p.Z == 0)
-        return warp_reduce_launch<KE, true, true>(sb, npairs, gout, p, g, 0, sm_count, st);
+        return warp_reduce_launch<KE, true, true>(sb, npairs, gout, p, g, 0, count_runs, sm_count,
+                                                  st);
     if (log2J >= 0)
-        return warp_reduce_launch<KE, false, true>(sb, npairs, gout, p, g, log2J, sm_count, st);
-    return warp_reduce_launch<KE, false, false>(sb, npairs, gout, p, g, 0, sm_count, st);
+        return warp_reduce_launch<KE, false, true>(sb, npairs, gout, p, g, log2J, count_runs,
+                                                   sm_count, st);
+    return warp_reduce_launch<KE, false, false>(sb, npairs, gout, p, g, 0, count_runs, sm_count,
+                                                st);
 }
 
 template <int VW, int KC, bool JPOW2, bool ZDIV>
 cudaError_t reduce_launch(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                          const DevParams& p, double* g, int log2J, int log2gs, int sm_count,
-                          cudaStream_t st) {
+                          const DevParams& p, double* g, int log2J, int log2gs, bool count_runs,
+                          int sm_count, cudaStream_t st) {
     const int gpc = kWarps * (32 >> log2gs);
     const size_t smem = sizeof(float) * (size_t)gpc * (size_t)p.L;
     const int64_t ntasks = (npairs + kPiece - 1) / kPiece;   // upper bound
     const int64_t work_blocks = (ntasks + gpc - 1) / gpc;
     const int grid = grid_for(k_range_reduce<VW, KC, JPOW2, ZDIV>, sm_count, work_blocks, smem);
     return launch_k(k_range_reduce<VW, KC, JPOW2, ZDIV>, dim3(grid), dim3(kThreads), smem, st,
-                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g, log2gs);
+                    sb.sorted_e, sb.stats, npairs, gout, p.d, p.Z, p.J, log2J, p.L, p.G, p.smask, g, log2gs,
+                    count_runs);
 }
 
 template <int VW, int KC>
 cudaError_t reduce_inst(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                        const DevParams& p, double* g, int log2gs, int sm_count,
+                        const DevParams& p, double* g, int log2gs, bool count_runs, int sm_count,
                         cudaStream_t st) {
     const int log2J = (p.J & (p.J - 1)) == 0 ? ceil_log2(p.J) : -1;
     if (p.d % p.Z == 0)
-        return reduce_launch<VW, KC, true, true>(sb, npairs, gout, p, g, 0, log2gs, sm_count, st);
+        return reduce_launch<VW, KC, true, true>(sb, npairs, gout, p, g, 0, log2gs, count_runs,
+                                                 sm_count, st);
     if (log2J >= 0)
-        return reduce_launch<VW, KC, true, false>(sb, npairs, gout, p, g, log2J, log2gs, sm_count,
-                                                  st);
-    return reduce_launch<VW, KC, false, false>(sb, npairs, gout, p, g, 0, log2gs, sm_count, st);
+        return reduce_launch<VW, KC, true, false>(sb, npairs, gout, p, g, log2J, log2gs,
+                                                  count_runs, sm_count, st);
+    return reduce_launch<VW, KC, false, false>(sb, npairs, gout, p, g, 0, log2gs, count_runs,
+                                               sm_count, st);
 }
 
 }  // namespace
@@ -1511,7 +1527,7 @@ cudaError_t launch_window_reduce(const SortedBuffers& sb, int64_t npairs, const 
     int grid = grid_for(k_async_reduce<kSinkOnce>, sm_count, blocks);
     cudaError_t e = launch_k(k_async_reduce<kSinkOnce>, dim3(grid), dim3(kThreads), 0, st,
                              sb.sorted_e, sb.stats, npairs, gout, p.G, p.smask,
-                             (double*)nullptr, ws, (const uint32_t*)nullptr);
+                             (double*)nullptr, ws, (const uint32_t*)nullptr, true);
     if (e != cudaSuccess) return e;
     grid = grid_for(k_window_combine, sm_count, blocks);
     return launch_k(k_window_combine, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e,
@@ -1542,8 +1558,8 @@ cudaError_t launch_sort_local(const SortedBuffers& sb, int64_t npairs, int J, ui
 }
 
 cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const float* gout,
-                                 const DevParams& p, double* g, bool local, int sm_count,
-                                 cudaStream_t st) {
+                                 const DevParams& p, double* g, bool local, bool count_runs,
+                                 int sm_count, cudaStream_t st) {
     if (local && !window_reduce_ok(p, gout)) return cudaErrorInvalidValue;
     // 32-element chunks tiling the rows: asynchronous shared-memory staging
     if (window_reduce_ok(p, gout)) {
@@ -1555,20 +1571,22 @@ cudaError_t launch_sorted_reduce(const SortedBuffers& sb, int64_t npairs, const 
         if (grid > 3 * sm_count) grid = 3 * sm_count;
         return launch_k(k_async_reduce<kSinkF64>, dim3(grid), dim3(kThreads), 0, st, sb.sorted_e,
                         sb.stats, npairs, gout, p.G, p.smask, g, WindowSink{},
-                        local ? (const uint32_t*)sb.segn : (const uint32_t*)nullptr);
+                        local ? (const uint32_t*)sb.segn : (const uint32_t*)nullptr, count_runs);
     }
     // blocks of 32+ elements: one warp per task, one element per lane
     if (p.L >= 32) {
-        if (p.L <= 32) return warp_reduce_inst<1>(sb, npairs, gout, p, g, sm_count, st);
-        if (p.L <= 64) return warp_reduce_inst<2>(sb, npairs, gout, p, g, sm_count, st);
-        if (p.L <= 128) return warp_reduce_inst<4>(sb, npairs, gout, p, g, sm_count, st);
+        if (p.L <= 32) return warp_reduce_inst<1>(sb, npairs, gout, p, g, count_runs, sm_count, st);
+        if (p.L <= 64) return warp_reduce_inst<2>(sb, npairs, gout, p, g, count_runs, sm_count, st);
+        if (p.L <= 128)
+            return warp_reduce_inst<4>(sb, npairs, gout, p, g, count_runs, sm_count, st);
     }
     const bool vec = (p.Z % 4 == 0) && (p.d % 4 == 0) && (((uintptr_t)gout & 15u) == 0);
     const int vw = vec ? 4 : 1;
     const int V = (p.L + vw - 1) / vw;
     const int log2gs = V <= 32 ? ceil_log2(V) : 5;
     const int kc = V <= 32 ? 1 : (1 << ceil_log2((V + 31) / 32));
-#define PSS_RD(VW, KC) return reduce_inst<VW, KC>(sb, npairs, gout, p, g, log2gs, sm_count, st)
+#define PSS_RD(VW, KC) \
+    return reduce_inst<VW, KC>(sb, npairs, gout, p, g, log2gs, count_runs, sm_count, st)
     if (vec) {
         switch (kc) {
             case 1: PSS_RD(4, 1);
