@@ -134,7 +134,8 @@ typedef enum {
      * pss_grad_noalloc does not wrap. */
     PSS_OPT_CIRCULAR = 7,
     /* Digit width of the sorted path's radix sort (used with
-     * PSS_OPT_DETERMINISTIC, and always above 2^22 block starts): 0 (default)
+     * PSS_OPT_DETERMINISTIC, and for a global sort above 2^22 block starts,
+     * see PSS_OPT_SORT_SCOPE): 0 (default)
      * sorts the bucket indices (bit width of R - 1) in as few passes of at
      * most 11 bits as possible; 4 to 11 forces that many bits per pass (more
      * passes).  The sort is stable, so the result does not depend on it. */
@@ -142,12 +143,14 @@ typedef enum {
     /* 1: run-to-run identical bits on the sorted path.  The sorted path then
      * sorts with the stable radix sort (see PSS_OPT_SORT_DIGIT_BITS), which
      * orders the contributions of every location by pair; the reduce sums
-     * them in that order, and the few run sums of an element meet in fp64
-     * (exact, hence in any order, unless their magnitudes span more than
-     * about 2^26).  0 (default): the faster counting sort, whose order within
-     * a location follows the GPU's scheduling (the sum is within the same
-     * bound, but low-order bits may differ between runs).  Above 2^22 block
-     * starts the radix sort is always used.  The atomic path is not affected. */
+     * them in that order; for 32-element chunks that tile the rows each
+     * element's additions then follow a fixed order (no atomics), for other
+     * shapes the few run sums of an element meet in fp64 (exact, hence in any
+     * order, unless their magnitudes span more than about 2^26).  0 (default):
+     * the faster counting or segment-local sort (PSS_OPT_SORT_SCOPE), whose
+     * order within a location follows the GPU's scheduling (the sum is within
+     * the same bound, but low-order bits may differ between runs).  The atomic
+     * path is not affected. */
     PSS_OPT_DETERMINISTIC = 9,
     /* How the sorted path (when not deterministic) groups the pairs by
      * location.  PSS_SORT_GLOBAL: one sort of all pairs (counting sort up to
